@@ -1,0 +1,210 @@
+/*
+ * dge.h -- C ABI of the Draft-Guided Eviction (DGE) score -> select -> compact
+ * pass on one GPU (sm_103a).
+ *
+ * The paper (Alg. 1) drafts k answer tokens on the full KV cache, then, once
+ * per layer and KV head: scores every past position with the observation
+ * queries (line B: the k draft queries; DGE-W: the base evictor's window), keeps
+ * the per-head budget (retention rule R_E: SnapKV top-B after max-pooling,
+ * PyramidKV per-layer budgets, H2O's accumulated attention, StreamingLLM's sinks
+ * + recency), and edits the cache keeping temporal order (App. E implementation
+ * notes: sort indices, gather [retained past] || [window + draft tail]).
+ *
+ * Conventions shared by every call:
+ *   - Caches are bf16, GQA ("kv_head") layout as in App. G: K, V are indexed
+ *     [layer][batch][kv_head][position][d] through the element strides of a
+ *     dge_tensor; d is contiguous.  Query rows are [layer][batch][q_head][row][d].
+ *     Query head g belongs to KV head g / (Hq / Hkv).
+ *   - A "unit" is one (layer, batch, kv_head).  Units are ordered
+ *     u = (layer * batch + b) * Hkv + h.
+ *   - Positions are int32 in [0, n).  Scored positions of a unit are [0, P) with
+ *     P = n - tail.  Scores are float32, [unit][P], contiguous.
+ *   - Packed outputs (idx, Kc, Vc) hold budgets[l] rows per unit, units in
+ *     order, so unit (l, b, h) starts at row
+ *       row_base(l) + (b * Hkv + h) * budgets[l],
+ *       row_base(l) = batch * Hkv * (budgets[0] + ... + budgets[l-1]).
+ *     Kc, Vc are [rows][d] bf16, contiguous.  idx rows are ascending positions.
+ *   - Every device pointer is caller-owned.  The library allocates no device
+ *     memory, keeps no device state between calls, and never synchronises the
+ *     caller's stream (except dge_get_device_status).  All work is enqueued on
+ *     `stream` (a cudaStream_t passed as void*; NULL = legacy default stream).
+ *   - Outputs must not alias inputs.
+ *   - Validation errors are returned before anything is enqueued.  Launch
+ *     failures return DGE_ERR_CUDA; dge_last_error() then holds the CUDA error
+ *     text for the calling thread.
+ */
+#ifndef DGE_H
+#define DGE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+enum {
+    DGE_OK = 0,
+    DGE_ERR_INVALID_ARG = 1,         /* null pointer, inconsistent sizes, bad budget */
+    DGE_ERR_UNSUPPORTED = 2,         /* head_dim, alignment or size outside what the kernels take */
+    DGE_ERR_WORKSPACE_TOO_SMALL = 3, /* ws_bytes below dge_workspace_size() */
+    DGE_ERR_CUDA = 4,                /* a CUDA launch or runtime call failed */
+    DGE_ERR_DEVICE_TIMEOUT = 5       /* a device-side bounded wait gave up (status word) */
+};
+
+/* Scoring variant (Alg. 1 line B and the retention rules of App. L). */
+enum {
+    DGE_VARIANT_SCORED = 0,    /* SnapKV / PyramidKV / DGE: the caller's m observation rows
+                                  per query head, row i at position n - m + i */
+    DGE_VARIANT_H2O = 1,       /* H2O accumulator: all n rows, row i at position i, causal */
+    DGE_VARIANT_STREAMING = 2  /* StreamingLLM: sinks + recency, no scores */
+};
+
+/* Pooling along positions before selection (App. B: max-pool, kernel 7). */
+enum {
+    DGE_POOL_NONE = 0,
+    DGE_POOL_MAX = 1,  /* max over the in-range cells of [j - r, j + r], r = kernel / 2 */
+    DGE_POOL_AVG = 2   /* sum over the in-range cells / kernel (zero padding) */
+};
+
+/*
+ * The eviction problem (Alg. 1 inputs: per-head budget B, draft length k,
+ * base evictor E with window w).
+ */
+typedef struct dge_problem {
+    int32_t num_layers;    /* L >= 1 (at most 256) */
+    int32_t batch;         /* b >= 1 */
+    int32_t num_q_heads;   /* Hq >= 1 */
+    int32_t num_kv_heads;  /* Hkv >= 1, divides Hq */
+    int32_t head_dim;      /* d: 64 or 128 */
+    int32_t obs_rows;      /* SCORED: m = w + k >= 1 rows per query head; ignored otherwise */
+    int64_t seq_len;       /* n >= 1, < 2^31: cache length incl. window and draft rows */
+    int32_t tail;          /* protected tail [n - tail, n): SCORED t (normally m), H2O the
+                              recent window; ignored by STREAMING */
+    int32_t sinks;         /* protected head [0, sinks) */
+    int32_t variant;       /* DGE_VARIANT_* */
+    int32_t pool;          /* DGE_POOL_* (SCORED only; H2O and STREAMING do not pool) */
+    int32_t pool_kernel;   /* odd, 1..31, when pool != NONE */
+    float scale;           /* logit scale; 0 means 1/sqrt(head_dim) */
+    const int32_t *budgets;/* HOST array [L]: kept rows per unit of layer l, counting the
+                              protected sinks and tail: sinks + tail <= budgets[l] <= n
+                              (STREAMING: sinks <= budgets[l] <= n) */
+} dge_problem;
+
+/* A bf16 tensor in device memory with element strides; d is contiguous.
+ * data must be 16-byte aligned and every stride a multiple of 8 elements. */
+typedef struct dge_tensor {
+    const void *data;
+    int64_t stride_layer, stride_batch, stride_head, stride_pos;
+} dge_tensor;
+
+/* Inputs and outputs of dge_evict / dge_score. */
+typedef struct dge_buffers {
+    dge_tensor K;        /* [L][b][Hkv][n][d] */
+    dge_tensor V;        /* [L][b][Hkv][n][d] (dge_evict only) */
+    dge_tensor Q;        /* [L][b][Hq][m][d] (SCORED) or [L][b][Hq][n][d] (H2O); unused by
+                            STREAMING */
+    float *scores;       /* [unit][P] final (pooled) scores; required by dge_score, optional
+                            (NULL) for dge_evict */
+    int32_t *idx;        /* packed kept positions (dge_evict) */
+    void *Kc;            /* packed [rows][d] bf16 (dge_evict) */
+    void *Vc;            /* packed [rows][d] bf16 (dge_evict) */
+} dge_buffers;
+
+/*
+ * Bytes of device workspace that dge_score / dge_evict need for this problem
+ * (for STREAMING only the 256-byte status region).  The workspace is
+ * caller-allocated, 256-byte aligned, and may be reused across calls on the
+ * same stream; its contents need no initialisation.  Its first 4 bytes are the
+ * device status word: dge_score and dge_evict clear it when they start,
+ * device-side checks set it, dge_get_device_status reads and clears it.
+ * Returns DGE_OK or DGE_ERR_INVALID_ARG / DGE_ERR_UNSUPPORTED.
+ */
+int dge_workspace_size(const dge_problem *p, size_t *bytes);
+
+/* Total rows of the packed outputs: batch * Hkv * sum(budgets). */
+int dge_packed_rows(const dge_problem *p, int64_t *rows);
+
+/*
+ * Scores (Alg. 1 line B; App. B): for every unit, over the stacked rows of its
+ * G = Hq / Hkv query heads,
+ *   raw[j] = sum_rows exp(s_rj - lse_r),  s_rj = scale * q_r . k_j  (j <= pos_r),
+ *   lse_r  = log sum_{j <= pos_r} exp(s_rj),
+ * for j in [0, P), then pooled along positions (SCORED only) and written to
+ * bufs->scores.  Uses bufs->K, bufs->Q, bufs->scores.  SCORED and H2O only.
+ */
+int dge_score(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+              void *stream);
+
+/*
+ * Retention (Alg. 1: I <- R_E(s, B - w); App. E: sort to keep temporal order).
+ * For every unit keeps [0, sinks), the budgets[l] - sinks - tail positions of
+ * [sinks, P) with the largest scores (equal scores: lower position first), and
+ * [P, n); writes them ascending to the packed idx.  STREAMING ignores scores
+ * (may be NULL) and keeps [0, sinks) and the last budgets[l] - sinks positions.
+ */
+int dge_select(const dge_problem *p, const float *scores, int32_t *idx, void *stream);
+
+/*
+ * Compaction (App. E: gather [retained past] || [window + draft tail]):
+ * Kc[r] = K[idx[r]], Vc[r] = V[idx[r]] for every packed row, a bit copy.
+ * idx values must lie in [0, n) (out-of-range rows are left unwritten and
+ * reported through dge_get_device_status as DGE_ERR_INVALID_ARG when a
+ * workspace is given; pass ws = NULL to skip that report).
+ */
+int dge_compact(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
+                const dge_tensor *V, void *Kc, void *Vc, void *ws, void *stream);
+
+/*
+ * The whole pass, score -> pool -> select -> compact, enqueued on one stream
+ * with no host synchronisation.  Writes bufs->idx, Kc, Vc and, when not NULL,
+ * bufs->scores.  STREAMING needs no workspace (ws may be NULL).
+ */
+int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+              void *stream);
+
+/*
+ * PyramidKV's per-layer past budgets (App. L): c = B - w, min = floor(c/20),
+ * max = 2c - min, steps = floor((max - min)/(L - 1)), out[l] = max - l*steps.
+ * These are past tokens only; add the protected tail to get dge budgets.
+ * Host only.  Needs L >= 2 and B > w.
+ */
+int dge_pyramid_budgets(int32_t B, int32_t w, int32_t L, int32_t *out);
+
+/*
+ * Synchronises `stream`, reads the device status word in `ws` (written by
+ * bounded device waits and device-side checks), clears it, and returns it
+ * (DGE_OK when nothing was reported).
+ */
+int dge_get_device_status(void *ws, void *stream);
+
+/*
+ * Kernel timing (tracing).  Between dge_profile_begin() and dge_profile_end(),
+ * every kernel the library enqueues is bracketed by two CUDA events on the
+ * call's stream (the GPU's own order is unchanged).  dge_profile_end() waits
+ * for those events, then writes up to `capacity` entries, one per kernel
+ * name, with the number of launches and their summed device time, and sets
+ * *count to the number of distinct kernels.  Host-side state is per process
+ * and guarded by a mutex; begin clears it.
+ */
+typedef struct dge_kernel_time {
+    char name[48];
+    int64_t launches;
+    double total_ms;
+} dge_kernel_time;
+
+int dge_profile_begin(void);
+int dge_profile_end(dge_kernel_time *out, int capacity, int *count);
+
+/* Static text for a status code. */
+const char *dge_status_string(int code);
+
+/* Text of the last CUDA error seen by a call on this thread ("" if none). */
+const char *dge_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DGE_H */

@@ -1,0 +1,162 @@
+"""Public Python entry points: allocate outputs with PyTorch, call the C ABI.
+
+Every function here marshals arguments and calls libdge; the computation runs
+in the library's CUDA kernels on the tensors' device and the current stream.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional, Sequence
+
+import torch
+
+from . import binding as B
+
+
+@dataclasses.dataclass
+class Problem:
+    """Shape and policy of one eviction pass (mirrors dge_problem)."""
+
+    L: int
+    b: int
+    Hq: int
+    Hkv: int
+    d: int
+    n: int
+    budgets: Sequence[int]
+    m: int = 0
+    tail: int = 0
+    sinks: int = 0
+    variant: int = B.DGE_VARIANT_SCORED
+    pool: int = B.DGE_POOL_NONE
+    pool_kernel: int = 1
+    scale: float = 0.0
+
+    def c(self) -> B.dge_problem:
+        return B.make_problem(L=self.L, b=self.b, Hq=self.Hq, Hkv=self.Hkv, d=self.d, n=self.n,
+                              m=self.m, tail=self.tail, sinks=self.sinks, variant=self.variant,
+                              pool=self.pool, pool_kernel=self.pool_kernel, scale=self.scale,
+                              budgets=self.budgets)
+
+    @property
+    def U(self) -> int:
+        return self.L * self.b * self.Hkv
+
+    @property
+    def P(self) -> int:
+        return self.n if self.variant == B.DGE_VARIANT_STREAMING else self.n - self.tail
+
+    def packed_rows(self) -> int:
+        return B.dge_packed_rows(self.c())
+
+    def workspace_bytes(self) -> int:
+        return B.dge_workspace_size(self.c())
+
+    def unit_row_offsets(self) -> list:
+        """First packed row of every unit, in unit order (layer, batch, kv head)."""
+        offs, acc = [], 0
+        for l in range(self.L):
+            for _ in range(self.b * self.Hkv):
+                offs.append(acc)
+                acc += self.budgets[l]
+        return offs
+
+
+def problem_from_workload(wl) -> Problem:
+    """The Problem of a synthetic workload (``inputs.Workload``)."""
+    return Problem(L=wl.L, b=wl.b, Hq=wl.Hq, Hkv=wl.Hkv, d=wl.d, n=wl.n, budgets=wl.budgets,
+                   m=wl.m, tail=wl.tail, sinks=wl.sinks, variant=wl.variant, pool=wl.pool,
+                   pool_kernel=wl.pool_kernel)
+
+
+def _stream(stream: Optional[torch.cuda.Stream]) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def workspace(p: Problem, device) -> torch.Tensor:
+    """A device workspace of dge_workspace_size() bytes (256-byte aligned)."""
+    nbytes = max(p.workspace_bytes(), 256)
+    ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
+    off = (-ws.data_ptr()) % 256
+    return ws[off:off + nbytes]
+
+
+def _check_cache(t: torch.Tensor, name: str) -> None:
+    if t.dtype != torch.bfloat16 or not t.is_cuda:
+        raise ValueError(f"{name} must be a bf16 CUDA tensor")
+
+
+def evict(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torch.Tensor] = None, *,
+          want_scores: bool = False, ws: Optional[torch.Tensor] = None,
+          out: Optional[dict] = None, stream=None) -> dict:
+    """dge_evict: the fused score -> pool -> select -> compact pass.
+
+    Returns {"idx", "Kc", "Vc", "scores"} (scores is None unless requested).
+    ``out`` may hold preallocated outputs with those keys.
+    """
+    _check_cache(K, "K")
+    _check_cache(V, "V")
+    dev = K.device
+    rows = p.packed_rows()
+    o = dict(out or {})
+    if o.get("idx") is None:
+        o["idx"] = torch.empty(rows, dtype=torch.int32, device=dev)
+    if o.get("Kc") is None:
+        o["Kc"] = torch.empty((rows, p.d), dtype=torch.bfloat16, device=dev)
+    if o.get("Vc") is None:
+        o["Vc"] = torch.empty((rows, p.d), dtype=torch.bfloat16, device=dev)
+    if want_scores and o.get("scores") is None:
+        o["scores"] = torch.empty((p.U, p.P), dtype=torch.float32, device=dev)
+    o.setdefault("scores", None)
+    if ws is None:
+        ws = workspace(p, dev)
+    bufs = B.dge_buffers(K=B.tensor_desc(K), V=B.tensor_desc(V), Q=B.tensor_desc(Q),
+                         scores=B.ptr(o["scores"]), idx=B.ptr(o["idx"]), Kc=B.ptr(o["Kc"]),
+                         Vc=B.ptr(o["Vc"]))
+    B.dge_evict(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
+    return o
+
+
+def score(p: Problem, K: torch.Tensor, Q: torch.Tensor, *, ws=None, stream=None) -> torch.Tensor:
+    """dge_score: final (pooled) scores [unit][P] in float32."""
+    _check_cache(K, "K")
+    _check_cache(Q, "Q")
+    scores = torch.empty((p.U, p.P), dtype=torch.float32, device=K.device)
+    if ws is None:
+        ws = workspace(p, K.device)
+    bufs = B.dge_buffers(K=B.tensor_desc(K), Q=B.tensor_desc(Q), scores=scores.data_ptr())
+    B.dge_score(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
+    return scores
+
+
+def select(p: Problem, scores: Optional[torch.Tensor], *, stream=None) -> torch.Tensor:
+    """dge_select: packed ascending kept positions (int32)."""
+    dev = scores.device if scores is not None else torch.device("cuda")
+    idx = torch.empty(p.packed_rows(), dtype=torch.int32, device=dev)
+    B.dge_select(p.c(), B.ptr(scores), idx.data_ptr(), _stream(stream))
+    return idx
+
+
+def compact(p: Problem, idx: torch.Tensor, K: torch.Tensor, V: torch.Tensor, *, ws=None,
+            stream=None) -> tuple:
+    """dge_compact: packed Kc, Vc gathered at idx."""
+    _check_cache(K, "K")
+    _check_cache(V, "V")
+    rows = p.packed_rows()
+    Kc = torch.empty((rows, p.d), dtype=torch.bfloat16, device=K.device)
+    Vc = torch.empty_like(Kc)
+    kd, vd = B.tensor_desc(K), B.tensor_desc(V)
+    B.dge_compact(p.c(), idx.data_ptr(), kd, vd, Kc.data_ptr(), Vc.data_ptr(),
+                  B.ptr(ws), _stream(stream))
+    return Kc, Vc
+
+
+def device_status(ws: torch.Tensor, stream=None) -> int:
+    """dge_get_device_status: sync the stream and read/clear the status word."""
+    return B.dge_get_device_status(ws.data_ptr(), _stream(stream))
+
+
+def pyramid_budgets(B_: int, w: int, L: int) -> list:
+    """PyramidKV per-layer past budgets (App. L)."""
+    return B.dge_pyramid_budgets(B_, w, L)

@@ -1,0 +1,517 @@
+// dge_api.cu -- the C ABI declared in include/dge.h: argument validation,
+// workspace layout and the launch sequence of the score -> select -> compact
+// pass.  Host code only; kernels live in score_mma.cu and select_compact.cu.
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <map>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace dge;
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+int cuda_fail(cudaError_t err, const char *where)
+{
+    snprintf(g_last_error, sizeof g_last_error, "%s: %s (%s)", where, cudaGetErrorName(err),
+             cudaGetErrorString(err));
+    return DGE_ERR_CUDA;
+}
+
+#define DGE_CHECK_CUDA(expr, where)                  \
+    do {                                             \
+        cudaError_t e_ = (expr);                     \
+        if (e_ != cudaSuccess)                       \
+            return cuda_fail(e_, where);             \
+    } while (0)
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// ---------------------------------------------------------------------------
+// Kernel timing: events around launches while profiling is on.
+struct ProfRecord {
+    const char *name;
+    cudaEvent_t start, stop;
+};
+
+struct Profiler {
+    std::mutex mu;
+    bool on = false;
+    std::vector<ProfRecord> records;
+    std::vector<cudaEvent_t> pool;
+
+    cudaEvent_t take()
+    {
+        if (!pool.empty()) {
+            cudaEvent_t e = pool.back();
+            pool.pop_back();
+            return e;
+        }
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess)
+            return nullptr;
+        return e;
+    }
+};
+
+Profiler &profiler()
+{
+    static Profiler p;
+    return p;
+}
+
+// Records a start event at construction and a stop event at destruction.
+class ProfScope {
+  public:
+    ProfScope(const char *name, cudaStream_t stream) : name_(name), stream_(stream)
+    {
+        Profiler &p = profiler();
+        std::lock_guard<std::mutex> lk(p.mu);
+        if (!p.on)
+            return;
+        start_ = p.take();
+        stop_ = p.take();
+        if (start_ && stop_ && cudaEventRecord(start_, stream_) == cudaSuccess)
+            active_ = true;
+    }
+    ~ProfScope()
+    {
+        if (!active_)
+            return;
+        Profiler &p = profiler();
+        std::lock_guard<std::mutex> lk(p.mu);
+        if (cudaEventRecord(stop_, stream_) == cudaSuccess)
+            p.records.push_back({name_, start_, stop_});
+    }
+
+  private:
+    const char *name_;
+    cudaStream_t stream_;
+    cudaEvent_t start_ = nullptr, stop_ = nullptr;
+    bool active_ = false;
+};
+
+#define DGE_LAUNCH(name, stream, expr)                                \
+    do {                                                              \
+        cudaError_t e_;                                               \
+        {                                                             \
+            ProfScope ps_(name, stream);                              \
+            e_ = (expr);                                              \
+        }                                                             \
+        if (e_ != cudaSuccess)                                        \
+            return cuda_fail(e_, name);                               \
+    } while (0)
+
+// Work decomposition and workspace layout of one problem.
+struct Plan {
+    Geometry g;
+    LayerTable layers;
+    int64_t packed_rows = 0;
+    int rows_per_block = 0;  // phase-1 row block (all rows for SCORED)
+    int chunk_keys = 0;      // phase-1 key chunk
+    int nchunks = 0;
+    size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, ws_bytes = 0;
+};
+
+constexpr int kScoredChunkKeys = 2048;
+constexpr int kH2ORowBlock = 128;
+
+int make_plan(const dge_problem *p, Plan &plan)
+{
+    if (!p || !p->budgets)
+        return DGE_ERR_INVALID_ARG;
+    const int64_t n = p->seq_len;
+    if (p->num_layers < 1 || p->num_layers > kMaxLayers || p->batch < 1 || p->num_q_heads < 1 ||
+        p->num_kv_heads < 1 || p->num_q_heads % p->num_kv_heads != 0 || n < 1 ||
+        n >= (int64_t)INT32_MAX || p->sinks < 0 || p->sinks > n)
+        return DGE_ERR_INVALID_ARG;
+    if (p->variant != DGE_VARIANT_SCORED && p->variant != DGE_VARIANT_H2O &&
+        p->variant != DGE_VARIANT_STREAMING)
+        return DGE_ERR_INVALID_ARG;
+    if (p->head_dim != 64 && p->head_dim != 128)
+        return DGE_ERR_UNSUPPORTED;
+    if (!isfinite(p->scale))
+        return DGE_ERR_INVALID_ARG;
+
+    Geometry &g = plan.g;
+    memset(&g, 0, sizeof g);
+    g.L = p->num_layers;
+    g.b = p->batch;
+    g.Hq = p->num_q_heads;
+    g.Hkv = p->num_kv_heads;
+    g.G = g.Hq / g.Hkv;
+    g.d = p->head_dim;
+    g.n = (int)n;
+    g.sinks = p->sinks;
+    g.variant = p->variant;
+    g.pool = DGE_POOL_NONE;
+    g.pool_kernel = 1;
+    g.U = (int64_t)g.L * g.b * g.Hkv;
+    const float scale = p->scale != 0.f ? p->scale : 1.f / sqrtf((float)g.d);
+    g.scale_log2 = scale * 1.4426950408889634f;
+
+    if (p->variant == DGE_VARIANT_STREAMING) {
+        g.tail = 0;
+        g.P = g.n;
+        g.m = 0;
+        g.R = 0;
+    } else {
+        if (p->tail < 0 || (int64_t)p->tail + p->sinks > n)
+            return DGE_ERR_INVALID_ARG;
+        g.tail = p->tail;
+        g.P = g.n - g.tail;
+        if (p->variant == DGE_VARIANT_SCORED) {
+            if (p->obs_rows < 1 || p->obs_rows > n)
+                return DGE_ERR_INVALID_ARG;
+            g.m = p->obs_rows;
+            if ((int64_t)g.G * g.m > kMaxRows)
+                return DGE_ERR_UNSUPPORTED;
+            g.R = g.G * g.m;
+            if (p->pool != DGE_POOL_NONE && p->pool != DGE_POOL_MAX && p->pool != DGE_POOL_AVG)
+                return DGE_ERR_INVALID_ARG;
+            if (p->pool != DGE_POOL_NONE &&
+                (p->pool_kernel < 1 || p->pool_kernel > 31 || p->pool_kernel % 2 == 0))
+                return DGE_ERR_INVALID_ARG;
+            g.pool = p->pool;
+            g.pool_kernel = p->pool == DGE_POOL_NONE ? 1 : p->pool_kernel;
+        } else {
+            g.m = 0;
+            if ((int64_t)g.G * n >= (int64_t)INT32_MAX)
+                return DGE_ERR_UNSUPPORTED;
+            g.R = (int)(g.G * n);
+        }
+    }
+
+    int64_t acc = 0;
+    for (int l = 0; l < g.L; ++l) {
+        const int32_t B = p->budgets[l];
+        const int64_t lo = (p->variant == DGE_VARIANT_STREAMING) ? g.sinks
+                                                                 : (int64_t)g.sinks + g.tail;
+        if (B < lo || B > n)
+            return DGE_ERR_INVALID_ARG;
+        plan.layers.budget[l] = B;
+        plan.layers.row_base[l] = acc;
+        acc += (int64_t)g.b * g.Hkv * B;
+    }
+    plan.packed_rows = acc;
+
+    if (p->variant == DGE_VARIANT_SCORED) {
+        plan.rows_per_block = g.R;
+        plan.chunk_keys = kScoredChunkKeys;
+    } else if (p->variant == DGE_VARIANT_H2O) {
+        plan.rows_per_block = kH2ORowBlock;
+        plan.chunk_keys = g.n;
+    }
+    size_t off = kStatusBytes;
+    if (p->variant != DGE_VARIANT_STREAMING) {
+        plan.nchunks = (g.n + plan.chunk_keys - 1) / plan.chunk_keys;
+        plan.off_partial = off;
+        off = align256(off + (size_t)g.U * g.R * plan.nchunks * sizeof(float2));
+        plan.off_lse = off;
+        off = align256(off + (size_t)g.U * g.R * sizeof(float));
+        plan.off_raw = off;
+        off = align256(off + (size_t)g.U * g.P * sizeof(float));
+        plan.off_pooled = off;
+        if (g.pool != DGE_POOL_NONE)
+            off = align256(off + (size_t)g.U * g.P * sizeof(float));
+    }
+    plan.ws_bytes = off;
+    return DGE_OK;
+}
+
+int check_tensor(const dge_tensor &t)
+{
+    if (!t.data)
+        return DGE_ERR_INVALID_ARG;
+    if (((uintptr_t)t.data & 15) != 0)
+        return DGE_ERR_UNSUPPORTED;
+    if (t.stride_layer < 0 || t.stride_batch < 0 || t.stride_head < 0 || t.stride_pos < 0)
+        return DGE_ERR_INVALID_ARG;
+    if ((t.stride_layer | t.stride_batch | t.stride_head | t.stride_pos) & 7)
+        return DGE_ERR_UNSUPPORTED;
+    return DGE_OK;
+}
+
+TensorDesc desc(const dge_tensor &t)
+{
+    TensorDesc d;
+    d.data = static_cast<const __nv_bfloat16 *>(t.data);
+    d.s_layer = t.stride_layer;
+    d.s_batch = t.stride_batch;
+    d.s_head = t.stride_head;
+    d.s_pos = t.stride_pos;
+    return d;
+}
+
+int check_ws(const Plan &plan, void *ws, size_t ws_bytes)
+{
+    if (!ws)
+        return DGE_ERR_INVALID_ARG;
+    if (((uintptr_t)ws & 255) != 0)
+        return DGE_ERR_UNSUPPORTED;
+    if (ws_bytes < plan.ws_bytes)
+        return DGE_ERR_WORKSPACE_TOO_SMALL;
+    return DGE_OK;
+}
+
+template <typename T>
+T *ws_at(void *ws, size_t off)
+{
+    return reinterpret_cast<T *>(static_cast<uint8_t *>(ws) + off);
+}
+
+// raw scores of every unit into the workspace.
+int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void *ws,
+                cudaStream_t stream)
+{
+    const Geometry &g = plan.g;
+    float2 *partial = ws_at<float2>(ws, plan.off_partial);
+    float *lse2 = ws_at<float>(ws, plan.off_lse);
+    float *raw = ws_at<float>(ws, plan.off_raw);
+    DGE_LAUNCH("lse_partial", stream, launch_lse_partial(K, Q, g, plan.rows_per_block, plan.chunk_keys, partial,
+                                      stream));
+    DGE_LAUNCH("combine_lse", stream, launch_combine_lse(partial, g.U * g.R, plan.nchunks, lse2, stream));
+    if (g.variant == DGE_VARIANT_H2O)
+        DGE_LAUNCH("colsum_keys", stream, launch_colsum_keys(K, Q, g, lse2, raw, stream));
+    else
+        DGE_LAUNCH("colsum_rows", stream, launch_colsum_rows(K, Q, g, kScoredChunkKeys, lse2, raw, stream));
+    return DGE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dge_workspace_size(const dge_problem *p, size_t *bytes)
+{
+    if (!bytes)
+        return DGE_ERR_INVALID_ARG;
+    Plan plan;
+    const int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    *bytes = plan.ws_bytes;
+    return DGE_OK;
+}
+
+int dge_packed_rows(const dge_problem *p, int64_t *rows)
+{
+    if (!rows)
+        return DGE_ERR_INVALID_ARG;
+    Plan plan;
+    const int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    *rows = plan.packed_rows;
+    return DGE_OK;
+}
+
+int dge_score(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+              void *stream_)
+{
+    Plan plan;
+    int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    if (plan.g.variant == DGE_VARIANT_STREAMING || !bufs || !bufs->scores)
+        return DGE_ERR_INVALID_ARG;
+    if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->Q)) != DGE_OK ||
+        (rc = check_ws(plan, ws, ws_bytes)) != DGE_OK)
+        return rc;
+    if (((uintptr_t)bufs->scores & 3) != 0)
+        return DGE_ERR_UNSUPPORTED;
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
+    if ((rc = run_scoring(plan, desc(bufs->K), desc(bufs->Q), ws, stream)) != DGE_OK)
+        return rc;
+    DGE_LAUNCH("pool", stream, launch_pool(ws_at<float>(ws, plan.off_raw), bufs->scores, plan.g.U, plan.g.P,
+                               plan.g.pool, plan.g.pool_kernel, stream));
+    return DGE_OK;
+}
+
+int dge_select(const dge_problem *p, const float *scores, int32_t *idx, void *stream_)
+{
+    Plan plan;
+    const int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    if (!idx || ((uintptr_t)idx & 3) != 0)
+        return DGE_ERR_INVALID_ARG;
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    if (plan.g.variant == DGE_VARIANT_STREAMING) {
+        DGE_LAUNCH("streaming", stream, launch_streaming_indices(plan.g, plan.layers, idx, stream));
+        return DGE_OK;
+    }
+    if (!scores || ((uintptr_t)scores & 3) != 0)
+        return DGE_ERR_INVALID_ARG;
+    DGE_LAUNCH("select", stream, launch_select(plan.g, plan.layers, scores, idx, stream));
+    return DGE_OK;
+}
+
+int dge_compact(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
+                const dge_tensor *V, void *Kc, void *Vc, void *ws, void *stream_)
+{
+    Plan plan;
+    int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    if (!idx || !K || !V || !Kc || !Vc)
+        return DGE_ERR_INVALID_ARG;
+    if ((rc = check_tensor(*K)) != DGE_OK || (rc = check_tensor(*V)) != DGE_OK)
+        return rc;
+    if (((uintptr_t)Kc & 15) || ((uintptr_t)Vc & 15) || ((uintptr_t)idx & 3) ||
+        ((uintptr_t)ws & 255))
+        return DGE_ERR_UNSUPPORTED;
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    DGE_LAUNCH("compact", stream, launch_compact(plan.g, plan.layers, idx, nullptr, desc(*K), desc(*V), Kc, Vc,
+                                  false, static_cast<uint32_t *>(ws), stream));
+    return DGE_OK;
+}
+
+int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+              void *stream_)
+{
+    Plan plan;
+    int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    if (!bufs || !bufs->idx || !bufs->Kc || !bufs->Vc)
+        return DGE_ERR_INVALID_ARG;
+    if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK)
+        return rc;
+    if (((uintptr_t)bufs->Kc & 15) || ((uintptr_t)bufs->Vc & 15) || ((uintptr_t)bufs->idx & 3) ||
+        ((uintptr_t)bufs->scores & 3))
+        return DGE_ERR_UNSUPPORTED;
+    const Geometry &g = plan.g;
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    if (g.variant == DGE_VARIANT_STREAMING) {
+        if (ws && ((uintptr_t)ws & 255))
+            return DGE_ERR_UNSUPPORTED;
+        if (ws)
+            DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
+        DGE_LAUNCH("compact", stream, launch_compact(g, plan.layers, nullptr, bufs->idx, desc(bufs->K),
+                                      desc(bufs->V), bufs->Kc, bufs->Vc, true,
+                                      static_cast<uint32_t *>(ws), stream));
+        return DGE_OK;
+    }
+    if ((rc = check_tensor(bufs->Q)) != DGE_OK || (rc = check_ws(plan, ws, ws_bytes)) != DGE_OK)
+        return rc;
+    DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
+    const TensorDesc K = desc(bufs->K), V = desc(bufs->V), Q = desc(bufs->Q);
+    if ((rc = run_scoring(plan, K, Q, ws, stream)) != DGE_OK)
+        return rc;
+    float *raw = ws_at<float>(ws, plan.off_raw);
+    const float *sel = raw;
+    if (g.pool != DGE_POOL_NONE) {
+        float *pooled = bufs->scores ? bufs->scores : ws_at<float>(ws, plan.off_pooled);
+        DGE_LAUNCH("pool", stream, launch_pool(raw, pooled, g.U, g.P, g.pool, g.pool_kernel, stream));
+        sel = pooled;
+    } else if (bufs->scores) {
+        DGE_CHECK_CUDA(cudaMemcpyAsync(bufs->scores, raw, (size_t)g.U * g.P * sizeof(float),
+                                       cudaMemcpyDeviceToDevice, stream),
+                       "scores copy");
+    }
+    DGE_LAUNCH("select", stream, launch_select(g, plan.layers, sel, bufs->idx, stream));
+    DGE_LAUNCH("compact", stream, launch_compact(g, plan.layers, bufs->idx, nullptr, K, V, bufs->Kc, bufs->Vc,
+                                  false, static_cast<uint32_t *>(ws), stream));
+    return DGE_OK;
+}
+
+int dge_pyramid_budgets(int32_t B, int32_t w, int32_t L, int32_t *out)
+{
+    if (!out || L < 2 || B <= w)
+        return DGE_ERR_INVALID_ARG;
+    const int32_t c = B - w;
+    const int32_t lo = c / 20;
+    const int32_t hi = 2 * c - lo;
+    const int32_t step = (hi - lo) / (L - 1);
+    for (int32_t l = 0; l < L; ++l)
+        out[l] = hi - l * step;
+    return DGE_OK;
+}
+
+int dge_get_device_status(void *ws, void *stream_)
+{
+    if (!ws)
+        return DGE_ERR_INVALID_ARG;
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    DGE_CHECK_CUDA(cudaStreamSynchronize(stream), "stream sync");
+    uint32_t v = 0;
+    DGE_CHECK_CUDA(cudaMemcpy(&v, ws, sizeof v, cudaMemcpyDeviceToHost), "status read");
+    DGE_CHECK_CUDA(cudaMemset(ws, 0, sizeof v), "status clear");
+    return (int)v;
+}
+
+const char *dge_status_string(int code)
+{
+    switch (code) {
+    case DGE_OK: return "ok";
+    case DGE_ERR_INVALID_ARG: return "invalid argument";
+    case DGE_ERR_UNSUPPORTED: return "unsupported (head_dim, alignment or size)";
+    case DGE_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case DGE_ERR_CUDA: return "CUDA error";
+    case DGE_ERR_DEVICE_TIMEOUT: return "device-side wait timed out";
+    default: return "unknown status";
+    }
+}
+
+const char *dge_last_error(void) { return g_last_error; }
+
+int dge_profile_begin(void)
+{
+    Profiler &p = profiler();
+    std::lock_guard<std::mutex> lk(p.mu);
+    for (auto &r : p.records) {
+        p.pool.push_back(r.start);
+        p.pool.push_back(r.stop);
+    }
+    p.records.clear();
+    p.on = true;
+    return DGE_OK;
+}
+
+int dge_profile_end(dge_kernel_time *out, int capacity, int *count)
+{
+    Profiler &p = profiler();
+    std::lock_guard<std::mutex> lk(p.mu);
+    p.on = false;
+    std::map<std::string, std::pair<int64_t, double>> acc;
+    std::vector<std::string> order;
+    int rc = DGE_OK;
+    for (auto &r : p.records) {
+        float ms = 0.f;
+        cudaError_t e = cudaEventSynchronize(r.stop);
+        if (e == cudaSuccess)
+            e = cudaEventElapsedTime(&ms, r.start, r.stop);
+        if (e != cudaSuccess && rc == DGE_OK)
+            rc = cuda_fail(e, "profile");
+        auto it = acc.find(r.name);
+        if (it == acc.end()) {
+            order.push_back(r.name);
+            it = acc.emplace(r.name, std::make_pair((int64_t)0, 0.0)).first;
+        }
+        it->second.first += 1;
+        it->second.second += ms;
+        p.pool.push_back(r.start);
+        p.pool.push_back(r.stop);
+    }
+    p.records.clear();
+    if (count)
+        *count = (int)order.size();
+    for (int i = 0; i < (int)order.size() && i < capacity && out; ++i) {
+        snprintf(out[i].name, sizeof out[i].name, "%s", order[i].c_str());
+        out[i].launches = acc[order[i]].first;
+        out[i].total_ms = acc[order[i]].second;
+    }
+    return rc;
+}
+
+}  // extern "C"

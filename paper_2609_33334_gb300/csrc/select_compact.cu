@@ -1,0 +1,332 @@
+// select_compact.cu -- pooling, per-unit top-B selection, and the K/V gather.
+//
+// Pooling (App. B, max-pool kernel 7; avg-pool for PyramidKV's workload) runs
+// along positions of [0, P).  Selection is the retention rule of Alg. 1
+// (I <- R_E(s, B - w)) with the kept set written in temporal order (App. E):
+// a radix select finds the exact (B - sinks - tail)-th largest score, then a
+// stable, position-ordered compaction keeps every larger score and the lowest
+// positions among the scores equal to it.  The gather copies K and V rows at
+// the kept positions into the packed compact cache (App. E).
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace dge {
+
+// ---------------------------------------------------------------------------
+// Pooling: out[u][j] = pool over raw[u][max(0, j - r) .. min(P - 1, j + r)].
+__global__ void pool_kernel(const float *__restrict__ raw, float *__restrict__ out, int64_t U,
+                            int P, int pool, int kernel)
+{
+    const int64_t total = U * (int64_t)P;
+    const int r = kernel / 2;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t u = i / P;
+        const int j = (int)(i - u * P);
+        const float *row = raw + u * P;
+        if (pool == DGE_POOL_NONE) {
+            out[i] = row[j];
+            continue;
+        }
+        const int lo = max(0, j - r), hi = min(P - 1, j + r);
+        if (pool == DGE_POOL_MAX) {
+            float m = -INFINITY;
+            for (int q = lo; q <= hi; ++q)
+                m = fmaxf(m, row[q]);
+            out[i] = m;
+        } else {
+            float s = 0.f;
+            for (int q = lo; q <= hi; ++q)
+                s += row[q];
+            out[i] = s / (float)kernel;
+        }
+    }
+}
+
+cudaError_t launch_pool(const float *raw, float *out, int64_t U, int P, int pool, int kernel,
+                        cudaStream_t stream)
+{
+    const int64_t total = U * (int64_t)P;
+    if (total == 0)
+        return cudaSuccess;
+    const int threads = 256;
+    const int64_t want = (total + threads - 1) / threads;
+    const int64_t blocks = want < 152 * 64 ? want : 152 * 64;
+    pool_kernel<<<(unsigned)blocks, threads, 0, stream>>>(raw, out, U, P, pool, kernel);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Selection.  One CTA of kSelThreads per unit.
+
+constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kSmemKeys = 53248;  // candidates held in shared memory (208 KiB)
+
+struct SelectParams {
+    Geometry g;
+    LayerTable layers;
+};
+
+__device__ __forceinline__ int64_t unit_row_base(const SelectParams &p, int64_t u, int &budget)
+{
+    int l, bb, h;
+    unit_coords(p.g, u, l, bb, h);
+    budget = p.layers.budget[l];
+    return p.layers.row_base[l] + (int64_t)(bb * p.g.Hkv + h) * budget;
+}
+
+// Block-wide exclusive scan of one flag per thread (ballot + warp totals).
+// Returns this thread's exclusive prefix and writes the block total to *total.
+__device__ __forceinline__ int block_flag_scan(bool flag, int *warp_tot, int *total)
+{
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const unsigned bal = __ballot_sync(0xffffffffu, flag);
+    const int in_warp = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0)
+        warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    if (warp == 0) {
+        const int v = lane < kSelWarps ? warp_tot[lane] : 0;
+        int incl = v;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int o = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off)
+                incl += o;
+        }
+        if (lane < kSelWarps)
+            warp_tot[kSelWarps + lane] = incl - v;  // exclusive offset of warp `lane`
+        if (lane == 31)
+            *total = incl;
+    }
+    __syncthreads();
+    const int r = warp_tot[kSelWarps + warp] + in_warp;
+    return r;
+}
+
+template <bool SMEM>
+__global__ void __launch_bounds__(kSelThreads)
+select_kernel(const float *__restrict__ scores, int32_t *__restrict__ idx, SelectParams p)
+{
+    extern __shared__ __align__(16) uint32_t skeys[];
+    __shared__ uint32_t hist[256];
+    __shared__ int warp_tot[2 * kSelWarps];
+    __shared__ int s_total[2];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_rank;
+
+    const int64_t u = blockIdx.x;
+    const Geometry &g = p.g;
+    int budget;
+    int32_t *out = idx + unit_row_base(p, u, budget);
+    const int P = g.P, s0 = g.sinks, tail = g.n - g.P;
+    const int C = P - s0;                    // candidates [s0, P)
+    const int keep = budget - s0 - tail;     // candidates to keep
+    const float *sc = scores + u * (int64_t)P + s0;
+
+    for (int j = threadIdx.x; j < s0; j += kSelThreads)
+        out[j] = j;
+    for (int j = threadIdx.x; j < tail; j += kSelThreads)
+        out[s0 + keep + j] = P + j;
+    if (keep <= 0)
+        return;
+    if (keep >= C) {
+        for (int j = threadIdx.x; j < C; j += kSelThreads)
+            out[s0 + j] = s0 + j;
+        return;
+    }
+
+    if (SMEM) {
+        for (int j = threadIdx.x; j < C; j += kSelThreads)
+            skeys[j] = float_key(sc[j]);
+        __syncthreads();
+    }
+    auto key_at = [&](int j) -> uint32_t { return SMEM ? skeys[j] : float_key(sc[j]); };
+
+    // Radix select, 8 bits per pass from the top: find T = the keep-th largest key.
+    uint32_t prefix = 0, mask = 0;
+    int rank = keep;  // 1-based rank of T among keys matching `prefix`, from the top
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        if (threadIdx.x < 256)
+            hist[threadIdx.x] = 0;
+        __syncthreads();
+        for (int j = threadIdx.x; j < C; j += kSelThreads) {
+            const uint32_t k = key_at(j);
+            if ((k & mask) == prefix)
+                atomicAdd(&hist[(k >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (threadIdx.x < 32) {
+            // Suffix sums over bins 255..0 by one warp: lane handles 8 bins.
+            const int lane = threadIdx.x;
+            uint32_t c[8];
+            uint32_t local = 0;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                c[q] = hist[255 - (lane * 8 + q)];
+                local += c[q];
+            }
+            uint32_t incl = local;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const uint32_t o = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off)
+                    incl += o;
+            }
+            uint32_t run = incl - local;  // keys in bins above this lane's first bin
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                if (run < (uint32_t)rank && run + c[q] >= (uint32_t)rank) {
+                    s_prefix = prefix | ((uint32_t)(255 - (lane * 8 + q)) << shift);
+                    s_rank = rank - (int)run;
+                }
+                run += c[q];
+            }
+        }
+        __syncthreads();
+        prefix = s_prefix;
+        rank = s_rank;
+        mask |= 255u << shift;
+        __syncthreads();
+    }
+    const uint32_t T = prefix;
+    const int need_eq = rank;  // keys equal to T to keep, lowest positions first
+
+    // Position-ordered compaction.
+    int sel_base = 0, eq_base = 0;
+    for (int base = 0; base < C; base += kSelThreads) {
+        const int j = base + threadIdx.x;
+        const uint32_t k = j < C ? key_at(j) : 0u;
+        const bool eq = j < C && k == T;
+        const int eq_rank = eq_base + block_flag_scan(eq, warp_tot, &s_total[0]);
+        const int eq_tot = s_total[0];
+        const bool sel = j < C && (k > T || (eq && eq_rank < need_eq));
+        const int pos = sel_base + block_flag_scan(sel, warp_tot, &s_total[1]);
+        const int sel_tot = s_total[1];
+        if (sel && pos < keep)
+            out[s0 + pos] = s0 + j;
+        eq_base += eq_tot;
+        sel_base += sel_tot;
+        __syncthreads();
+    }
+}
+
+cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const float *scores,
+                          int32_t *idx, cudaStream_t stream)
+{
+    SelectParams p;
+    p.g = g;
+    p.layers = layers;
+    const int C = g.P - g.sinks;
+    if (C <= kSmemKeys) {
+        const size_t smem = (size_t)max(C, 1) * sizeof(uint32_t);
+        if (smem > 48 * 1024) {
+            cudaError_t err = cudaFuncSetAttribute(
+                select_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+            if (err != cudaSuccess)
+                return err;
+        }
+        select_kernel<true><<<(unsigned)g.U, kSelThreads, smem, stream>>>(scores, idx, p);
+    } else {
+        select_kernel<false><<<(unsigned)g.U, kSelThreads, 0, stream>>>(scores, idx, p);
+    }
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// StreamingLLM indices: [0, sinks) then the last budget - sinks positions.
+__global__ void streaming_index_kernel(int32_t *__restrict__ idx, SelectParams p)
+{
+    const int64_t u = blockIdx.x;
+    int budget;
+    int32_t *out = idx + unit_row_base(p, u, budget);
+    const int s0 = p.g.sinks, n = p.g.n;
+    for (int r = threadIdx.x; r < budget; r += blockDim.x)
+        out[r] = r < s0 ? r : n - budget + r;
+}
+
+cudaError_t launch_streaming_indices(const Geometry &g, const LayerTable &layers, int32_t *idx,
+                                     cudaStream_t stream)
+{
+    SelectParams p;
+    p.g = g;
+    p.layers = layers;
+    streaming_index_kernel<<<(unsigned)g.U, 256, 0, stream>>>(idx, p);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Gather: Kc[row] = K[idx[row]], Vc[row] = V[idx[row]], 16-byte vectors.
+// Block = (unit, row block of kGatherRows); implicit = StreamingLLM indices
+// computed in place (and written to idx).
+constexpr int kGatherRows = 64;
+
+template <int D>
+__global__ void __launch_bounds__(256)
+compact_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__ idx_out, TensorDesc K,
+               TensorDesc V, __nv_bfloat16 *__restrict__ Kc, __nv_bfloat16 *__restrict__ Vc,
+               SelectParams p, int nrb, int implicit, uint32_t *status)
+{
+    constexpr int TPR = D / 8;             // threads per row (16 B each)
+    constexpr int RPI = 256 / TPR;          // rows per iteration
+    const int64_t u = blockIdx.x / nrb;
+    const int rb = (int)(blockIdx.x % nrb);
+    int l, bb, h;
+    unit_coords(p.g, u, l, bb, h);
+    int budget;
+    const int64_t base = unit_row_base(p, u, budget);
+    const int r_lo = rb * kGatherRows;
+    const int r_hi = min(r_lo + kGatherRows, budget);
+    const __nv_bfloat16 *Ku = kv_unit_ptr(K, l, bb, h);
+    const __nv_bfloat16 *Vu = kv_unit_ptr(V, l, bb, h);
+    const int part = threadIdx.x % TPR;
+    for (int r = r_lo + threadIdx.x / TPR; r < r_hi; r += RPI) {
+        int pos;
+        if (implicit) {
+            pos = r < p.g.sinks ? r : p.g.n - budget + r;
+            if (part == 0 && idx_out)
+                idx_out[base + r] = pos;
+        } else {
+            pos = idx_in[base + r];
+        }
+        if (pos < 0 || pos >= p.g.n) {
+            if (part == 0)
+                set_status(status, DGE_ERR_INVALID_ARG);
+            continue;
+        }
+        const int4 kv = *reinterpret_cast<const int4 *>(Ku + (int64_t)pos * K.s_pos + part * 8);
+        const int4 vv = *reinterpret_cast<const int4 *>(Vu + (int64_t)pos * V.s_pos + part * 8);
+        *reinterpret_cast<int4 *>(Kc + (base + r) * D + part * 8) = kv;
+        *reinterpret_cast<int4 *>(Vc + (base + r) * D + part * 8) = vv;
+    }
+}
+
+cudaError_t launch_compact(const Geometry &g, const LayerTable &layers, const int32_t *idx_in,
+                           int32_t *idx_out, const TensorDesc &K, const TensorDesc &V, void *Kc,
+                           void *Vc, bool implicit, uint32_t *status, cudaStream_t stream)
+{
+    SelectParams p;
+    p.g = g;
+    p.layers = layers;
+    int maxb = 0;
+    for (int l = 0; l < g.L; ++l)
+        maxb = max(maxb, layers.budget[l]);
+    const int nrb = (maxb + kGatherRows - 1) / kGatherRows;
+    if (nrb == 0)
+        return cudaSuccess;
+    const int64_t blocks = g.U * nrb;
+    if (g.d == 128)
+        compact_kernel<128><<<(unsigned)blocks, 256, 0, stream>>>(
+            idx_in, idx_out, K, V, static_cast<__nv_bfloat16 *>(Kc),
+            static_cast<__nv_bfloat16 *>(Vc), p, nrb, implicit ? 1 : 0, status);
+    else
+        compact_kernel<64><<<(unsigned)blocks, 256, 0, stream>>>(
+            idx_in, idx_out, K, V, static_cast<__nv_bfloat16 *>(Kc),
+            static_cast<__nv_bfloat16 *>(Vc), p, nrb, implicit ? 1 : 0, status);
+    return cudaGetLastError();
+}
+
+}  // namespace dge

@@ -1,0 +1,194 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+Small cases compare every unit element by element; the full-size workloads
+run in the launch configuration bench.py times and are checked on sampled
+units that the oracle computes one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_33334_gb300 import _build, api, inputs
+from parity import compare_unit, oracle_units, unit_list, unit_rows
+
+pytestmark = pytest.mark.gpu
+
+WL = inputs.WORKLOADS
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    _build.build()
+    oracle.build()
+
+
+def run(wl, want_scores=True, tens=None, **kw):
+    tens = tens or inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    Q = tens["Q"] if wl.variant != inputs.STREAMING else None
+    out = api.evict(p, tens["K"], tens["V"], Q, want_scores=want_scores and
+                    wl.variant != inputs.STREAMING, **kw)
+    torch.cuda.synchronize()
+    return tens, out
+
+
+def check_all(wl, tens, out, units=None):
+    units = unit_list(wl) if units is None else units
+    refs = oracle_units(wl, tens, units)
+    diffs = 0
+    for (l, b, h) in units:
+        diffs += compare_unit(wl, out, tens, l, b, h, ref=refs[(l, b, h)])
+    return diffs
+
+
+# --- small cases: every unit ------------------------------------------------------------
+
+def test_tiny_workload_matches_oracle():
+    wl = WL["c1_tiny"]
+    tens, out = run(wl)
+    check_all(wl, tens, out)
+
+
+SMALL = {
+    # reduced-n / reduced-L variants of the larger workloads (ragged tails included)
+    "c2_small": WL["c2_8b_8k"].with_(L=2, n=3000),
+    "c3_small": WL["c3_8b_32k_pyramid"].with_(L=3, b=2, n=4500, budgets=(900, 610, 301),
+                                              n_spans=8),
+    "c4_small": WL["c4_h2o_8k"].with_(L=1, b=2, n=1000, budgets=(200,)),
+    "c5_small": WL["c5_70b_128k"].with_(L=1, n=5000, budgets=(700,), n_spans=16),
+    "slm_small": WL["c5_slm"].with_(L=2, n=5000, budgets=(700, 300), n_spans=0),
+    # edge cases
+    "keep_none": WL["c1_tiny"].with_(budgets=(10,)),                   # B == tail
+    "keep_all": WL["c1_tiny"].with_(budgets=(1024,)),                  # B == n
+    "one_row": WL["c1_tiny"].with_(Hq=2, Hkv=2, w=1, k=0, budgets=(40,), n_spans=0),
+    "short_cache": WL["c1_tiny"].with_(n=37, budgets=(20,), n_spans=0),
+    "sinks_scored": WL["c1_tiny"].with_(sinks=4, budgets=(100,)),
+    "no_pool": WL["c1_tiny"].with_(pool=inputs.POOL_NONE, pool_kernel=1),
+    "avg_pool_31": WL["c1_tiny"].with_(pool=inputs.POOL_AVG, pool_kernel=31),
+    "max_pool_3_d128": WL["c1_tiny"].with_(d=128, pool_kernel=3),
+    "gqa8_ragged": WL["c1_tiny"].with_(Hq=16, Hkv=2, n=2117, budgets=(333,)),
+    "h2o_tiny": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=4, Hkv=2, d=64, n=300, budgets=(100,)),
+    "slm_keep_all": WL["c5_slm"].with_(L=1, n=300, Hq=8, Hkv=2, budgets=(300,), n_spans=0),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_small_cases_match_oracle(name):
+    wl = SMALL[name]
+    tens, out = run(wl)
+    check_all(wl, tens, out)
+
+
+def test_strided_views_match_contiguous():
+    """K/V/Q as strided views of larger buffers give the same result."""
+    wl = WL["c1_tiny"].with_(L=2, b=2, budgets=(128, 64))
+    tens = inputs.make_inputs(wl, device="cuda")
+    big = {}
+    for k, t in tens.items():
+        shape = list(t.shape)
+        shape[3] += 24          # extra positions / rows per head
+        buf = torch.zeros(shape[:4] + [shape[4] + 64], dtype=t.dtype, device="cuda")
+        view = buf[:, :, :, 5:5 + t.shape[3], 32:32 + t.shape[4]]
+        view.copy_(t)
+        big[k] = view
+    p = api.problem_from_workload(wl)
+    a = api.evict(p, tens["K"], tens["V"], tens["Q"], want_scores=True)
+    b = api.evict(p, big["K"], big["V"], big["Q"], want_scores=True)
+    torch.cuda.synchronize()
+    for k in ("idx", "Kc", "Vc", "scores"):
+        assert torch.equal(a[k], b[k]), k
+
+
+def test_runs_are_bit_identical():
+    """Re-runs reproduce every output byte (deterministic reductions)."""
+    wl = SMALL["c3_small"]
+    tens, a = run(wl)
+    _, b = run(wl, tens=tens)
+    for k in ("idx", "Kc", "Vc", "scores"):
+        assert torch.equal(a[k], b[k]), k
+
+
+def test_separate_calls_match_fused():
+    """dge_score -> dge_select -> dge_compact equals dge_evict."""
+    wl = SMALL["c2_small"]
+    tens, fused = run(wl)
+    p = api.problem_from_workload(wl)
+    s = api.score(p, tens["K"], tens["Q"])
+    idx = api.select(p, s)
+    Kc, Vc = api.compact(p, idx, tens["K"], tens["V"])
+    torch.cuda.synchronize()
+    assert torch.equal(s, fused["scores"])
+    assert torch.equal(idx, fused["idx"])
+    assert torch.equal(Kc, fused["Kc"]) and torch.equal(Vc, fused["Vc"])
+
+
+def test_select_on_oracle_scores_is_exact():
+    """With identical float32 scores on both sides, the kept set is identical."""
+    wl = WL["c1_tiny"].with_(L=2, budgets=(128, 200))
+    rng = np.random.default_rng(3)
+    p = api.problem_from_workload(wl)
+    # plateaus of equal values (as max-pooling makes) plus random values
+    base = rng.random((p.U, p.P)).astype(np.float32)
+    base[:, 100:140] = 0.75
+    base[:, 500:520] = base[:, 500:501]
+    scores = torch.from_numpy(base).cuda()
+    idx = api.select(p, scores).cpu().numpy()
+    for (l, b, h) in unit_list(wl):
+        u = (l * wl.b + b) * wl.Hkv + h
+        want = oracle.select(base[u].astype(np.float64), wl.n, wl.sinks, wl.tail, wl.budgets[l])
+        r0, r1 = unit_rows(wl, l, b, h)
+        np.testing.assert_array_equal(idx[r0:r1], want)
+
+
+def test_compact_out_of_range_index_reports_status():
+    """A bad index is skipped and reported through the status word, not a fault."""
+    wl = WL["c1_tiny"]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    idx = torch.arange(p.packed_rows(), dtype=torch.int32, device="cuda")
+    idx[5] = wl.n + 3
+    ws = api.workspace(p, "cuda")
+    ws.zero_()
+    Kc, Vc = api.compact(p, idx, tens["K"], tens["V"], ws=ws)
+    assert api.device_status(ws) == 1
+    assert api.device_status(ws) == 0          # reading clears it
+    good = idx.clone()
+    good[5] = 5
+    Kc2, _ = api.compact(p, good, tens["K"], tens["V"])
+    torch.cuda.synchronize()
+    assert torch.equal(Kc[:5], Kc2[:5]) and torch.equal(Kc[6:], Kc2[6:])
+
+
+# --- full-size workloads, sampled units --------------------------------------------------
+
+FULL = ["c2_8b_8k", "c3_8b_32k_pyramid", "c4_h2o_8k", "c5_70b_128k", "c5_slm"]
+
+
+def sample_units(wl, k=3, seed=0):
+    U = wl.L * wl.b * wl.Hkv
+    rng = np.random.default_rng(seed)
+    picks = {0, U - 1} | set(rng.choice(U, size=min(k, U), replace=False).tolist())
+    return sorted(picks)
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled_units(name):
+    wl = WL[name]
+    tens, out = run(wl)
+    units = unit_list(wl, sample_units(wl, k=2 if name in ("c4_h2o_8k", "c5_70b_128k") else 3))
+    check_all(wl, tens, out, units)
+    # properties over every unit: ascending, exact length, tail kept
+    idx = out["idx"].cpu().numpy()
+    start = 0
+    for l in range(wl.L):
+        B = wl.budgets[l]
+        blk = idx[start:start + wl.b * wl.Hkv * B].reshape(-1, B)
+        start += wl.b * wl.Hkv * B
+        assert np.all(np.diff(blk, axis=1) > 0)
+        if wl.tail:
+            assert np.all(blk[:, -wl.tail:] == np.arange(wl.n - wl.tail, wl.n))
+    del tens, out
+    torch.cuda.empty_cache()
