@@ -138,6 +138,29 @@ int dge_score(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
               void *stream);
 
 /*
+ * dge_score without a workspace argument and without allocating anything, for
+ * callers that are not allowed to allocate device memory: code embedded in a
+ * serving runtime that owns the whole device-memory plan and rejects any
+ * allocation on its request path, or code that must not call cudaMalloc /
+ * cudaFree because those can synchronise the whole device while other streams
+ * are running.  The paper has no counterpart; this is a deployment convenience.
+ *
+ * Scratch is a fixed device array built into the library,
+ * DGE_NOALLOC_SCRATCH_BYTES (32 MiB); every GPU that loads the library holds
+ * it until the process exits.  A problem whose dge_workspace_size() exceeds it
+ * is rejected with DGE_ERR_WORKSPACE_TOO_SMALL before anything is enqueued
+ * (dge_last_error() then states both sizes).  The first call on each device
+ * looks up the array's device address with that device current, so make that
+ * first call before any stream capture.  Every call uses the same array and it
+ * keeps the previous call's contents (the call itself clears what must start
+ * at zero), so calls that can overlap on the GPU -- on different streams or
+ * from different host threads -- race; serialise them.  Inputs, outputs and
+ * results are those of dge_score.
+ */
+#define DGE_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+int dge_score_noalloc(const dge_problem *p, const dge_buffers *bufs, void *stream);
+
+/*
  * Retention (Alg. 1: I <- R_E(s, B - w); App. E: sort to keep temporal order).
  * For every unit keeps [0, sinks), the budgets[l] - sinks - tail positions of
  * [sinks, P) with the largest scores (equal scores: lower position first), and

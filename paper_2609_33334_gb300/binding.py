@@ -66,6 +66,7 @@ _SIGS = {
     "dge_workspace_size": [_P, POINTER(c_size_t)],
     "dge_packed_rows": [_P, POINTER(c_int64)],
     "dge_score": [_P, _B, c_void_p, c_size_t, c_void_p],
+    "dge_score_noalloc": [_P, _B, c_void_p],
     "dge_select": [_P, c_void_p, c_void_p, c_void_p],
     "dge_compact": [_P, c_void_p, _T, _T, c_void_p, c_void_p, c_void_p, c_void_p],
     "dge_evict": [_P, _B, c_void_p, c_size_t, c_void_p],
@@ -122,6 +123,12 @@ def dge_packed_rows(p: dge_problem) -> int:
 def dge_score(p: dge_problem, bufs: dge_buffers, ws: int, ws_bytes: int, stream: int) -> None:
     _check("dge_score", _lib().dge_score(ctypes.byref(p), ctypes.byref(bufs), ws, ws_bytes,
                                          stream))
+
+
+def dge_score_noalloc(p: dge_problem, bufs: dge_buffers, stream: int) -> None:
+    """dge_score with the library's built-in scratch (no workspace, nothing allocated)."""
+    _check("dge_score_noalloc", _lib().dge_score_noalloc(ctypes.byref(p), ctypes.byref(bufs),
+                                                         stream))
 
 
 def dge_select(p: dge_problem, scores: int, idx: int, stream: int) -> None:

@@ -288,6 +288,11 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
 
 }  // namespace
 
+void dge::record_error_text(const char *text)
+{
+    snprintf(g_last_error, sizeof g_last_error, "%s", text);
+}
+
 extern "C" {
 
 int dge_workspace_size(const dge_problem *p, size_t *bytes)

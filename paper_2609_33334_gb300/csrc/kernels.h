@@ -28,4 +28,7 @@ cudaError_t launch_compact(const Geometry &g, const LayerTable &layers, const in
                            int32_t *idx_out, const TensorDesc &K, const TensorDesc &V, void *Kc,
                            void *Vc, bool implicit, uint32_t *status, cudaStream_t stream);
 
+// Stores `text` as the calling thread's dge_last_error() message.
+void record_error_text(const char *text);
+
 }  // namespace dge
