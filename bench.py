@@ -105,8 +105,8 @@ def kernel_bytes(wl, name):
     P = wl.n - wl.tail
     rows = wl.b * wl.Hkv * sum(wl.budgets)
     row_bytes = wl.d * 2
-    if name == "lse_partial":
-        return U * wl.n * row_bytes              # K read once
+    if name in ("lse_partial", "score_tc"):
+        return U * wl.n * row_bytes              # K read once (score_tc: both phases)
     if name in ("colsum_rows", "colsum_keys"):
         return U * P * row_bytes                 # K[0, P) read once
     if name == "compact":

@@ -220,6 +220,22 @@ typedef struct dge_kernel_time {
 int dge_profile_begin(void);
 int dge_profile_end(dge_kernel_time *out, int capacity, int *count);
 
+/*
+ * Cycle accounting of the tensor-core scoring kernel (tracing).  When `buffer`
+ * (device memory, caller-owned) is not NULL, every CTA of later launches writes
+ * per-role sums of SM clock cycles into it, slot-major: entry
+ * slot * DGE_TRACE_LEN + cta.  Slots: 0 MMA waiting for the query block, 1 MMA
+ * waiting for key tiles, 2 MMA waiting for a free accumulator, 3 MMA issuing, 4 MMA
+ * committing, 5 MMA total, 6 producer waiting for a query buffer, 7 producer waiting
+ * for a key stage, 8 producer total, 9 first epilogue warp waiting for accumulators,
+ * 10 (unused), 11 its phase-1 task ends, 12 its phase-2 task starts, 13 its exchange
+ * waits, 14 its total, 15 tiles issued.  `cta` is ignored.  `bytes` must cover the
+ * slots; pass NULL to stop.  Host-side state, per process.
+ */
+#define DGE_TRACE_SLOTS 16
+#define DGE_TRACE_LEN 4096
+int dge_trace_set(void *buffer, size_t bytes, int cta);
+
 /* Static text for a status code. */
 const char *dge_status_string(int code);
 

@@ -75,6 +75,7 @@ _SIGS = {
     "dge_status_string": [c_int],
     "dge_last_error": [],
     "dge_profile_begin": [],
+    "dge_trace_set": [c_void_p, c_size_t, c_int],
     "dge_profile_end": [POINTER(dge_kernel_time), c_int, POINTER(c_int)],
 }
 
@@ -175,6 +176,14 @@ def dge_profile_end(capacity: int = 32) -> list:
     _check("dge_profile_end", _lib().dge_profile_end(arr, capacity, ctypes.byref(count)))
     return [(arr[i].name.decode(), arr[i].launches, arr[i].total_ms)
             for i in range(min(count.value, capacity))]
+
+
+TRACE_SLOTS, TRACE_LEN = 16, 4096
+
+
+def dge_trace_set(buffer: int, nbytes: int, cta: int = 0) -> None:
+    """Record per-tile clock stamps of one CTA of the tensor-core scoring kernel."""
+    _check("dge_trace_set", _lib().dge_trace_set(buffer, nbytes, cta))
 
 
 # --- marshalling helpers --------------------------------------------------------------

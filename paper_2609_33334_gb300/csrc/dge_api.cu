@@ -3,6 +3,7 @@
 // pass.  Host code only; kernels live in score_mma.cu and select_compact.cu.
 #include <math.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <map>
@@ -118,7 +119,9 @@ struct Plan {
     int rows_per_block = 0;  // phase-1 row block (all rows for SCORED)
     int chunk_keys = 0;      // phase-1 key chunk
     int nchunks = 0;
-    size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, ws_bytes = 0;
+    TcPlan tc = {};          // tensor-core path decomposition (SCORED only)
+    size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, off_count = 0,
+           off_ready = 0, ws_bytes = 0;
 };
 
 constexpr int kScoredChunkKeys = 2048;
@@ -213,8 +216,16 @@ int make_plan(const dge_problem *p, Plan &plan)
     size_t off = kStatusBytes;
     if (p->variant != DGE_VARIANT_STREAMING) {
         plan.nchunks = (g.n + plan.chunk_keys - 1) / plan.chunk_keys;
+        // The partial region serves both scoring paths (the larger of the two layouts).
+        size_t part_bytes = (size_t)g.U * g.R * plan.nchunks * sizeof(float2);
+        if (p->variant == DGE_VARIANT_SCORED) {
+            plan.tc = tc_plan(g);
+            const size_t tc_bytes = (size_t)g.U * g.R * plan.tc.nchunks * sizeof(float);
+            if (tc_bytes > part_bytes)
+                part_bytes = tc_bytes;
+        }
         plan.off_partial = off;
-        off = align256(off + (size_t)g.U * g.R * plan.nchunks * sizeof(float2));
+        off = align256(off + part_bytes);
         plan.off_lse = off;
         off = align256(off + (size_t)g.U * g.R * sizeof(float));
         plan.off_raw = off;
@@ -222,6 +233,10 @@ int make_plan(const dge_problem *p, Plan &plan)
         plan.off_pooled = off;
         if (g.pool != DGE_POOL_NONE)
             off = align256(off + (size_t)g.U * g.P * sizeof(float));
+        plan.off_count = off;
+        off = align256(off + (size_t)g.U * sizeof(uint32_t));
+        plan.off_ready = off;
+        off = align256(off + (size_t)g.U * sizeof(uint32_t));
     }
     plan.ws_bytes = off;
     return DGE_OK;
@@ -268,6 +283,16 @@ T *ws_at(void *ws, size_t off)
     return reinterpret_cast<T *>(static_cast<uint8_t *>(ws) + off);
 }
 
+// Which scoring kernels to use: the tcgen05 path when the problem and device allow it,
+// unless DGE_SCORE_KERNEL=mma asks for the warp-level path.
+bool want_tc(const Geometry &g)
+{
+    const char *env = getenv("DGE_SCORE_KERNEL");
+    if (env && strcmp(env, "mma") == 0)
+        return false;
+    return tc_supported(g);
+}
+
 // raw scores of every unit into the workspace.
 int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void *ws,
                 cudaStream_t stream)
@@ -276,6 +301,35 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
     float2 *partial = ws_at<float2>(ws, plan.off_partial);
     float *lse2 = ws_at<float>(ws, plan.off_lse);
     float *raw = ws_at<float>(ws, plan.off_raw);
+    if (g.variant == DGE_VARIANT_SCORED && want_tc(g)) {
+        uint32_t *count = ws_at<uint32_t>(ws, plan.off_count);
+        uint32_t *ready = ws_at<uint32_t>(ws, plan.off_ready);
+        DGE_CHECK_CUDA(cudaMemsetAsync(count, 0, (size_t)g.U * sizeof(uint32_t), stream),
+                       "counter clear");
+        DGE_CHECK_CUDA(cudaMemsetAsync(ready, 0, (size_t)g.U * sizeof(uint32_t), stream),
+                       "flag clear");
+        TcBuffers tb;
+        tb.part = reinterpret_cast<float *>(partial);
+        tb.lse2 = lse2;
+        tb.raw = raw;
+        tb.count = count;
+        tb.ready = ready;
+        tb.status = static_cast<uint32_t *>(ws);
+        bool encoded = false;
+        DGE_LAUNCH("score_tc", stream,
+                   launch_score_tc(K, Q, g, plan.tc, tb, stream, &encoded));
+        if (encoded) {
+            // Units whose row sums left fp32's safe range (ready == 2) are recomputed
+            // with the running-maximum kernels; every other unit returns at once.
+            DGE_LAUNCH("recompute_lse", stream,
+                       launch_lse_partial(K, Q, g, g.R, g.n, partial, stream, ready));
+            DGE_LAUNCH("recompute_combine", stream,
+                       launch_combine_lse(partial, g.U * g.R, 1, lse2, stream, ready, g.R));
+            DGE_LAUNCH("recompute_colsum", stream,
+                       launch_colsum_rows(K, Q, g, g.P, lse2, raw, stream, ready));
+            return DGE_OK;
+        }
+    }
     DGE_LAUNCH("lse_partial", stream, launch_lse_partial(K, Q, g, plan.rows_per_block, plan.chunk_keys, partial,
                                       stream));
     DGE_LAUNCH("combine_lse", stream, launch_combine_lse(partial, g.U * g.R, plan.nchunks, lse2, stream));
@@ -469,6 +523,15 @@ const char *dge_status_string(int code)
 }
 
 const char *dge_last_error(void) { return g_last_error; }
+
+int dge_trace_set(void *buffer, size_t bytes, int cta)
+{
+    if (buffer && (bytes < (size_t)DGE_TRACE_SLOTS * DGE_TRACE_LEN * sizeof(uint64_t) ||
+                   ((uintptr_t)buffer & 7) || cta < 0))
+        return DGE_ERR_INVALID_ARG;
+    tc_set_trace(static_cast<unsigned long long *>(buffer), cta);
+    return DGE_OK;
+}
 
 int dge_profile_begin(void)
 {

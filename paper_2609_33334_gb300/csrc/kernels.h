@@ -5,15 +5,41 @@
 
 namespace dge {
 
-// Scoring (score_mma.cu).
+// Scoring on the warp-level tensor core path (score_mma.cu).  `only` (nullable, [U])
+// restricts the work to units whose entry equals kUnitRecompute.
+constexpr uint32_t kUnitRecompute = 2;
 cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int rows_per_block, int chunk_keys, float2 *partial,
-                               cudaStream_t stream);
+                               cudaStream_t stream, const uint32_t *only = nullptr);
 cudaError_t launch_combine_lse(const float2 *partial, int64_t total_rows, int nchunks,
-                               float *lse2, cudaStream_t stream);
+                               float *lse2, cudaStream_t stream, const uint32_t *only = nullptr,
+                               int rows_per_unit = 1);
 cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int chunk_keys, const float *lse2, float *raw,
-                               cudaStream_t stream);
+                               cudaStream_t stream, const uint32_t *only = nullptr);
+
+// Scoring on the tcgen05 path (score_tc.cu).
+struct TcPlan {
+    int r_pad, nslab, chunk_keys, nchunks, kstages;
+    size_t smem;
+};
+struct TcBuffers {
+    float *part;       // [U][nchunks][R] row sums of each key chunk
+    float *lse2;       // [U][R]
+    float *raw;        // [U][P]
+    uint32_t *count;   // [U], zero before the launch
+    uint32_t *ready;   // [U], zero before the launch; 1 = lse ready, 2 = recompute
+    uint32_t *status;
+};
+bool tc_supported(const Geometry &g);
+// Trace buffer of the tensor-core scoring kernel (see dge_trace_set); nullptr = off.
+void tc_set_trace(unsigned long long *buffer, int cta);
+TcPlan tc_plan(const Geometry &g);
+// Both phases in one launch.  *encoded is false when the tensors cannot be described
+// to TMA (nothing is launched then).
+cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                            const TcPlan &plan, const TcBuffers &buf, cudaStream_t stream,
+                            bool *encoded);
 cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                const float *lse2, float *raw, cudaStream_t stream);
 

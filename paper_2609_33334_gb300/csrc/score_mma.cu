@@ -112,13 +112,16 @@ __device__ __forceinline__ int max_row_position(const Geometry &g, int r0, int r
 template <int D, int MAX_NTW>
 __global__ void __launch_bounds__(kThreads)
 lse_partial_kernel(TensorDesc K, TensorDesc Q, Geometry g, int rows_per_block, int nrb,
-                   int chunk_keys, int nchunks, float2 *__restrict__ partial)
+                   int chunk_keys, int nchunks, float2 *__restrict__ partial,
+                   const uint32_t *__restrict__ only)
 {
     extern __shared__ __align__(16) uint8_t smem[];
     const int64_t bid = blockIdx.x;
     const int chunk = (int)(bid % nchunks);
     const int rb = (int)((bid / nchunks) % nrb);
     const int64_t u = bid / ((int64_t)nchunks * nrb);
+    if (only && only[u] != kUnitRecompute)
+        return;
     int l, bb, h;
     unit_coords(g, u, l, bb, h);
     const int r0 = rb * rows_per_block;
@@ -220,10 +223,13 @@ lse_partial_kernel(TensorDesc K, TensorDesc Q, Geometry g, int rows_per_block, i
 
 // lse_r = M + log2(sum_c z_c 2^{m_c - M}) over the chunks of row r.
 __global__ void combine_lse_kernel(const float2 *__restrict__ partial, int64_t total_rows,
-                                   int nchunks, float *__restrict__ lse2)
+                                   int nchunks, float *__restrict__ lse2,
+                                   const uint32_t *__restrict__ only, int rows_per_unit)
 {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= total_rows)
+        return;
+    if (only && only[i / rows_per_unit] != kUnitRecompute)
         return;
     const float2 *p = partial + i * nchunks;
     float M = neg_inf();
@@ -241,11 +247,14 @@ __global__ void combine_lse_kernel(const float2 *__restrict__ partial, int64_t t
 template <int D, int MAX_NTW>
 __global__ void __launch_bounds__(kThreads)
 colsum_rows_kernel(TensorDesc K, TensorDesc Q, Geometry g, int chunk_keys, int nchunks,
-                   const float *__restrict__ lse2, float *__restrict__ raw)
+                   const float *__restrict__ lse2, float *__restrict__ raw,
+                   const uint32_t *__restrict__ only)
 {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ float sCol[kThreads / 32][kTileKeys];
     const int64_t u = blockIdx.x / nchunks;
+    if (only && only[u] != kUnitRecompute)
+        return;
     const int chunk = (int)(blockIdx.x % nchunks);
     int l, bb, h;
     unit_coords(g, u, l, bb, h);
@@ -463,7 +472,7 @@ static cudaError_t prepare(KernelT kernel, size_t smem)
 
 cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int rows_per_block, int chunk_keys, float2 *partial,
-                               cudaStream_t stream)
+                               cudaStream_t stream, const uint32_t *only)
 {
     const int nrb = (g.R + rows_per_block - 1) / rows_per_block;
     const int nchunks = (g.n + chunk_keys - 1) / chunk_keys;
@@ -477,7 +486,8 @@ cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const G
                          err = prepare(k, smem);
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
-                                 K, Q, g, rows_per_block, nrb, chunk_keys, nchunks, partial);
+                                 K, Q, g, rows_per_block, nrb, chunk_keys, nchunks, partial,
+                                 only);
                              err = cudaGetLastError();
                          })
     } else {
@@ -486,7 +496,8 @@ cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const G
                          err = prepare(k, smem);
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
-                                 K, Q, g, rows_per_block, nrb, chunk_keys, nchunks, partial);
+                                 K, Q, g, rows_per_block, nrb, chunk_keys, nchunks, partial,
+                                 only);
                              err = cudaGetLastError();
                          })
     }
@@ -494,18 +505,19 @@ cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const G
 }
 
 cudaError_t launch_combine_lse(const float2 *partial, int64_t total_rows, int nchunks,
-                               float *lse2, cudaStream_t stream)
+                               float *lse2, cudaStream_t stream, const uint32_t *only,
+                               int rows_per_unit)
 {
     const int threads = 256;
     const int64_t blocks = (total_rows + threads - 1) / threads;
     combine_lse_kernel<<<(unsigned)blocks, threads, 0, stream>>>(partial, total_rows, nchunks,
-                                                                  lse2);
+                                                                  lse2, only, rows_per_unit);
     return cudaGetLastError();
 }
 
 cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int chunk_keys, const float *lse2, float *raw,
-                               cudaStream_t stream)
+                               cudaStream_t stream, const uint32_t *only)
 {
     const int nchunks = (g.P + chunk_keys - 1) / chunk_keys;
     const int rows_pad = (g.R + 7) & ~7;
@@ -518,7 +530,7 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
                          err = prepare(k, smem);
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
-                                 K, Q, g, chunk_keys, nchunks, lse2, raw);
+                                 K, Q, g, chunk_keys, nchunks, lse2, raw, only);
                              err = cudaGetLastError();
                          })
     } else {
@@ -527,7 +539,7 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
                          err = prepare(k, smem);
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
-                                 K, Q, g, chunk_keys, nchunks, lse2, raw);
+                                 K, Q, g, chunk_keys, nchunks, lse2, raw, only);
                              err = cudaGetLastError();
                          })
     }

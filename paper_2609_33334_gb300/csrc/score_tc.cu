@@ -1,0 +1,1001 @@
+// score_tc.cu -- the attention-score pass on the 5th-generation tensor cores.
+//
+// Same quantities as score_mma.cu (Alg. 1 line B; App. B; App. G), in base 2:
+//   x_rj = log2(e) * scale * q_r . k_j,  lse_r = log2 sum_{j <= pos_r} 2^{x_rj},
+//   raw_j = sum_r 2^{x_rj - lse_r}.
+//
+// One persistent CTA per SM, warp-specialised:
+//   warp 0      TMA producer: the unit's stacked query block (5-D box, G heads x m
+//               rows) and 128-key tiles of K, 128-byte swizzled, into a ring;
+//   warp 1      MMA issuer: D[128 keys x R_pad rows] = K_tile . Q^T with
+//               tcgen05.mma (M = 128, N = R_pad <= 256, bf16 -> fp32) into one of
+//               two TMEM accumulators; also owns the TMEM allocation;
+//   warps 2-9   epilogue: two warpgroups, each thread one key (TMEM lane), each
+//               warpgroup half of the row columns.
+// Work items are (unit, key chunk).  Step t of CTA s runs phase 1 of item
+// t*S + s (per-row sums 2^x over the chunk, reduced across the 128 keys at the
+// end) and then phase 2 of item (t-1)*S + s (2^{x - lse} summed over rows per
+// key), so phase 2 re-reads a chunk this CTA streamed one step earlier, from L2.
+// The last phase-1 task of a unit merges the chunk sums into lse and publishes
+// a ready flag; phase-2 tasks wait for it (bounded).  Row sums use no running
+// maximum: fp32 holds 2^x for |x| < 126, and a unit whose sums leave
+// [2^-60, 2^126) is flagged (ready = 2) and recomputed by the warp-level path.
+//
+// Every wait is bounded: on expiry the CTA records DGE_ERR_DEVICE_TIMEOUT in the
+// status word, stops issuing work, waits (bounded) for its own copies and MMAs,
+// frees TMEM and returns.
+#include <cuda.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc_ptx.cuh"
+
+namespace dge {
+
+namespace {
+
+constexpr int kTile = 128;
+constexpr int kEpiWG = 3;                 // epilogue warpgroups
+constexpr int kEpiWarps = 4 * kEpiWG;
+constexpr int kEpiWarp0 = 4;              // epilogue warps are 4 .. 15 (aligned warpgroups)
+constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
+// Registers per thread after reallocation: warpgroup 0 (producer, MMA, two idle warps)
+// gives up registers to the epilogue warpgroups.  The block launches with 512 threads x 128
+// registers; 4*32*56 + 12*32*152 is exactly that.
+constexpr int kRegsLaunch = 128, kRegsControl = 56, kRegsEpilogue = 152;
+static_assert(4 * 32 * kRegsControl + kEpiWarps * 32 * kRegsEpilogue <= kThreads * kRegsLaunch,
+              "register split");
+constexpr int kMaxGroups = 3;             // 16-column groups per epilogue warpgroup
+constexpr int kBarAllEpi = 1 + kEpiWG;    // named barrier of all epilogue warps (1..: one per WG)
+constexpr int kMaxKStages = 4;
+constexpr int kAccBufs = 3;               // TMEM accumulators
+constexpr int kTmemCols = 512;
+constexpr int kSlabBytes = kTile * 128;  // 128 rows x 64 bf16
+constexpr uint32_t kReadyOk = 1, kReadyBad = 2;
+
+// Barrier slots.
+constexpr int kBarKFull = 0, kBarKEmpty = 4, kBarQFull = 8, kBarQEmpty = 10, kBarAccFull = 12,
+              kBarAccEmpty = 15, kBarDrain = 18, kBarXFull = 19, kBarXEmpty = 21, kBarRedFull = 23,
+              kBarRedEmpty = 25, kBarLseFull = 27, kBarLseEmpty = 29, kNumBars = 31;
+constexpr int kBarCoord = 1 + kEpiWG + 1;  // named barrier of the two coordinator warps
+constexpr int kCoordThreads = 64;          // warps 2 and 3
+// Flag slots (ints): abort, last-arrival, wait result, out-of-range, then the parity of
+// the last arm of every key stage and query buffer (-1 = never armed) for the drain.
+constexpr int kFlagAbort = 0, kFlagLast = 1, kFlagWait = 2, kFlagBad = 3, kFlagKArm = 4,
+              kFlagQArm = 8;
+
+struct TcArgs {
+    Geometry g;
+    int r_pad, nslab, kstages;
+    int acc_stride;    // TMEM columns between accumulator buffers
+    int chunk_keys, nchunks;
+    int64_t items;
+    int ng[kEpiWG];    // 16-column groups of each epilogue warpgroup
+    int gbase[kEpiWG]; // first group of each epilogue warpgroup
+    int64_t steps;
+    float *part;       // [U][nchunks][R]
+    float *lse2;       // [U][R]
+    float *raw;        // [U][P]
+    uint32_t *count;   // [U]
+    uint32_t *ready;   // [U]
+    uint32_t *status;
+    unsigned long long timeout_ns;
+    unsigned long long *trace;  // see dge_trace_set; nullptr = off
+    int trace_cta;
+};
+
+// Cycle accounting (see dge_trace_set): per-role sums of SM clock cycles, written once per
+// CTA at the end into trace[slot * DGE_TRACE_LEN + blockIdx.x].
+enum TraceSlot {
+    kTrMmaWaitQ = 0, kTrMmaWaitK, kTrMmaWaitAcc, kTrMmaIssue, kTrMmaCommit, kTrMmaTotal,
+    kTrProdWaitQ, kTrProdWaitK, kTrProdTotal, kTrEpiWaitAcc, kTrEpiTiles, kTrEpiP1End,
+    kTrEpiP2Start, kTrEpiExchange, kTrEpiTotal, kTrTiles
+};
+
+__device__ __forceinline__ void trace_put(const TcArgs &a, int slot, long long v)
+{
+    if (a.trace && blockIdx.x < DGE_TRACE_LEN)
+        a.trace[slot * DGE_TRACE_LEN + blockIdx.x] = (unsigned long long)v;
+}
+
+struct Task {
+    int phase;
+    int64_t u;
+    int chunk, k_lo, k_hi, ntiles;
+};
+
+// Task j (0: phase 1, 1: phase 2) of step t for this CTA: phase 1 of item t*S + s, phase 2
+// of item (t-1)*S + s.  False when there is none (or it covers no keys).
+__device__ __forceinline__ bool get_task(const TcArgs &a, int64_t t, int j, Task &T)
+{
+    const int64_t S = gridDim.x, s = blockIdx.x;
+    int64_t item;
+    if (j == 0) {
+        item = t * S + s;
+        T.phase = 1;
+    } else {
+        if (t < 1)
+            return false;
+        item = (t - 1) * S + s;
+        T.phase = 2;
+    }
+    if (item >= a.items)
+        return false;
+    T.u = item / a.nchunks;
+    T.chunk = (int)(item % a.nchunks);
+    T.k_lo = T.chunk * a.chunk_keys;
+    const int end = T.phase == 1 ? a.g.n : a.g.P;
+    T.k_hi = min(T.k_lo + a.chunk_keys, end);
+    if (T.k_lo >= T.k_hi)
+        return false;
+    T.ntiles = (T.k_hi - T.k_lo + kTile - 1) / kTile;
+    return true;
+}
+
+struct Smem {
+    uint8_t *q;          // [2][nslab][r_pad * 128]
+    uint8_t *k;          // [kstages][nslab][kSlabBytes]
+    uint64_t *bar;       // [kNumBars]
+    uint32_t *tmem;      // allocation result
+    int *flag;           // [16]
+    float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
+    float *sL;           // [2][256] -lse of the rows of a phase-2 task (padding: -inf)
+    int *sLbad;          // [2] that task's unit is recomputed elsewhere
+    float *xch;          // [2][kEpiWG - 1][128] phase-2 column sums of warpgroups 1..
+};
+
+__host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
+{
+    return 1024                                   // alignment slack
+           + (size_t)2 * nslab * r_pad * 128      // query buffers
+           + (size_t)kstages * nslab * kSlabBytes // key ring
+           + kNumBars * 8 + 16 + 64               // barriers, tmem holder, flags
+           + (2 * kEpiWG * 4 * kMaxGroups * 16 + 2 * 256 + 2 * (kEpiWG - 1) * 128 + 4) * 4;
+}
+
+__device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
+{
+    // Offsets from the shared-memory symbol itself, so every pointer stays a shared-space
+    // pointer (32-bit addressing) rather than a generic one.
+    const uint32_t base = ptx::smem_addr(raw);
+    uint32_t off = ((base + 1023u) & ~1023u) - base;
+    Smem s;
+    s.q = raw + off;
+    off += (uint32_t)(2 * nslab * r_pad * 128);
+    s.k = raw + off;
+    off += (uint32_t)(kstages * nslab * kSlabBytes);
+    s.bar = reinterpret_cast<uint64_t *>(raw + off);
+    off += kNumBars * 8;
+    s.tmem = reinterpret_cast<uint32_t *>(raw + off);
+    off += 16;
+    s.flag = reinterpret_cast<int *>(raw + off);
+    off += 64;
+    s.red = reinterpret_cast<float *>(raw + off);
+    off += 2 * kEpiWG * 4 * kMaxGroups * 16 * 4;
+    s.sL = reinterpret_cast<float *>(raw + off);
+    off += 2 * 256 * 4;
+    s.sLbad = reinterpret_cast<int *>(raw + off);
+    off += 16;
+    s.xch = reinterpret_cast<float *>(raw + off);
+    return s;
+}
+
+// Bounded wait on an mbarrier phase.  Returns false when the CTA has aborted or the
+// wait outlived the timeout (then it aborts the CTA and records the status).
+__device__ bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *flag, const TcArgs &a)
+{
+    uint64_t t0 = 0;
+    uint32_t spins = 0;
+    while (!ptx::mbar_try_wait(bar, parity)) {
+        if ((++spins & 63) == 0) {
+            if (flag[kFlagAbort])
+                return false;
+            const uint64_t now = ptx::globaltimer();
+            if (t0 == 0) {
+                t0 = now;
+            } else if (now - t0 > a.timeout_ns) {
+                flag[kFlagAbort] = 1;
+                set_status(a.status, DGE_ERR_DEVICE_TIMEOUT);
+                return false;
+            }
+        }
+    }
+    return true;
+}
+
+// Bounded wait that ignores the abort flag (teardown drains).
+__device__ void drain_bar(uint64_t *bar, uint32_t parity, unsigned long long limit_ns)
+{
+    const uint64_t t0 = ptx::globaltimer();
+    while (!ptx::mbar_try_wait(bar, parity))
+        if (ptx::globaltimer() - t0 > limit_ns)
+            return;
+}
+
+// In-place sums over the 32 lanes of a warp, for 32 per-lane values held as two
+// 16-value groups a (columns 0..15) and b (16..31): afterwards a[0] of lane l holds
+// the total of column l.  Each step halves the values a lane keeps: the lane whose
+// bit o is set keeps the upper half, its partner the lower half.
+__device__ __forceinline__ void transpose_sum32(float (&a)[16], float (&b)[16], int lane)
+{
+    const bool up16 = (lane & 16) != 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const float send = up16 ? a[i] : b[i];
+        const float keep = up16 ? b[i] : a[i];
+        a[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+    }
+#pragma unroll
+    for (int o = 8; o >= 1; o >>= 1) {
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < o; ++i) {
+            const float send = upper ? a[i] : a[i + o];
+            const float keep = upper ? a[i + o] : a[i];
+            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+}
+
+// Same for one 16-value group: lanes l and l ^ 16 both end with column l & 15 in a[0].
+__device__ __forceinline__ void transpose_sum16(float (&a)[16], int lane)
+{
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+        a[i] += __shfl_xor_sync(0xffffffffu, a[i], 16);
+#pragma unroll
+    for (int o = 8; o >= 1; o >>= 1) {
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < o; ++i) {
+            const float send = upper ? a[i] : a[i + o];
+            const float keep = upper ? a[i + o] : a[i];
+            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+}
+
+// Visibility of the 16 columns cb .. cb+15 to `key` on tiles that reach the observation
+// rows' own positions: row r sits at first_causal + r % m and sees keys up to there.
+__device__ __forceinline__ uint32_t causal_mask(int key, int first_causal, int cb, int m)
+{
+    uint32_t mask = 0;
+#pragma unroll
+    for (int c = 0; c < 16; ++c)
+        mask |= (key <= first_causal + (cb + c) % m ? 1u : 0u) << c;
+    return mask;
+}
+
+// Phase 1 for one 16-column group: z[c] += 2^{x_c} (masked columns add nothing).
+__device__ __forceinline__ void rows_add(float (&z)[16], const float (&v)[16], float s2, bool valid,
+                                         bool causal, int key, int first_causal, int cb, int m)
+{
+    if (!valid)
+        return;
+    if (!causal) {
+        const float2 sc = make_float2(s2, s2);
+#pragma unroll
+        for (int c = 0; c < 16; c += 2) {
+            const float2 x = __fmul2_rn(make_float2(v[c], v[c + 1]), sc);
+            const float2 acc = __fadd2_rn(make_float2(z[c], z[c + 1]),
+                                          make_float2(ex2(x.x), ex2(x.y)));
+            z[c] = acc.x;
+            z[c + 1] = acc.y;
+        }
+    } else {
+        const uint32_t mask = causal_mask(key, first_causal, cb, m);
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+            const float e = ex2(v[c] * s2);
+            z[c] += ((mask >> c) & 1u) ? e : 0.f;
+        }
+    }
+}
+
+// Phase 2 for one 16-column group: adds 2^{x_c - lse_c} over the group's rows into the
+// pair accumulator.  nL holds -lse (padded columns: -inf).
+__device__ __forceinline__ void col_add(float2 &acc, const float (&v)[16], const float (&nL)[16],
+                                        float s2, bool causal, int key, int first_causal, int cb,
+                                        int m)
+{
+    if (!causal) {
+        const float2 sc = make_float2(s2, s2);
+#pragma unroll
+        for (int c = 0; c < 16; c += 2) {
+            const float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc,
+                                        make_float2(nL[c], nL[c + 1]));
+            acc = __fadd2_rn(acc, make_float2(ex2(x.x), ex2(x.y)));
+        }
+    } else {
+        const uint32_t mask = causal_mask(key, first_causal, cb, m);
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+            const float p = ex2(v[c] * s2 + nL[c]);
+            acc.x += ((mask >> c) & 1u) ? p : 0.f;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
+                const TcArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    const Smem sm = carve(smem_raw, a.r_pad, a.nslab, a.kstages);
+    volatile int *flag = sm.flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const Geometry &g = a.g;
+    const uint32_t q_slab_bytes = (uint32_t)a.r_pad * 128;
+
+    // ---- set-up -------------------------------------------------------------------
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < a.kstages; ++i) {
+            ptx::mbar_init(&sm.bar[kBarKFull + i], 1);
+            ptx::mbar_init(&sm.bar[kBarKEmpty + i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(&sm.bar[kBarQFull + i], 1);
+            ptx::mbar_init(&sm.bar[kBarQEmpty + i], 1);
+        }
+        for (int i = 0; i < kAccBufs; ++i) {
+            ptx::mbar_init(&sm.bar[kBarAccFull + i], 1);
+            ptx::mbar_init(&sm.bar[kBarAccEmpty + i], kEpiWarps);
+        }
+        ptx::mbar_init(&sm.bar[kBarDrain], 1);
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(&sm.bar[kBarXFull + i], 4 * (kEpiWG - 1));
+            ptx::mbar_init(&sm.bar[kBarXEmpty + i], 4);
+            ptx::mbar_init(&sm.bar[kBarRedFull + i], kEpiWarps);
+            ptx::mbar_init(&sm.bar[kBarRedEmpty + i], 1);
+            ptx::mbar_init(&sm.bar[kBarLseFull + i], 1);
+            ptx::mbar_init(&sm.bar[kBarLseEmpty + i], kEpiWarps);
+        }
+        flag[kFlagAbort] = 0;
+        flag[kFlagLast] = 0;
+        flag[kFlagWait] = 0;
+        flag[kFlagBad] = 0;
+        for (int i = 0; i < kMaxKStages; ++i)
+            flag[kFlagKArm + i] = -1;
+        flag[kFlagQArm] = flag[kFlagQArm + 1] = -1;
+        ptx::fence_mbar_init();
+    }
+    // Query rows R .. r_pad-1 are never written by TMA: zero them once so the padded
+    // accumulator columns are exactly 0.
+    {
+        const int pad_rows = a.r_pad - g.R;
+        const int words = pad_rows * 128 / 16;
+        for (int b = 0; b < 2; ++b)
+            for (int s = 0; s < a.nslab; ++s) {
+                int4 *base = reinterpret_cast<int4 *>(sm.q + ((size_t)b * a.nslab + s) * q_slab_bytes +
+                                                      (size_t)g.R * 128);
+                for (int i = threadIdx.x; i < words; i += blockDim.x)
+                    base[i] = make_int4(0, 0, 0, 0);
+            }
+        ptx::fence_proxy_async_smem();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(sm.tmem, kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem_base = *sm.tmem;
+
+    if (warp < kEpiWarp0) {
+        ptx::regs_dec<kRegsControl>();
+    if (warp == 0) {
+        // ---- TMA producer ---------------------------------------------------------------
+        if (lane == 0) {
+            ptx::prefetch_tmap(&tmK);
+            ptx::prefetch_tmap(&tmQ);
+            // Phase-1 tiles stay in L2 for the phase-2 re-read one step later; the re-read
+            // marks them first to go.
+            const uint64_t keep = ptx::make_policy_evict_last();
+            const uint64_t drop = ptx::make_policy_evict_first();
+            int ks = 0, qb = 0;
+            uint32_t kph = 0, qph = 0;
+            long long cy_wq = 0, cy_wk = 0;
+            const long long cy0 = clock64();
+            bool ok = true;
+            for (int64_t t = 0; ok && t <= a.steps; ++t)
+                for (int j = 0; ok && j < 2; ++j) {
+                    Task T;
+                    if (!get_task(a, t, j, T))
+                        continue;
+                    int l, bb, h;
+                    unit_coords(g, T.u, l, bb, h);
+                    long long c0 = clock64();
+                    if (!wait_bar(&sm.bar[kBarQEmpty + qb], qph ^ 1, flag, a)) {
+                        ok = false;
+                        break;
+                    }
+                    cy_wq += clock64() - c0;
+                    ptx::mbar_arrive_expect_tx(&sm.bar[kBarQFull + qb],
+                                               (uint32_t)a.nslab * 128u * (uint32_t)g.R);
+                    flag[kFlagQArm + qb] = (int)qph;
+                    for (int s = 0; s < a.nslab; ++s)
+                        ptx::tma_load_5d_hint(sm.q + ((size_t)qb * a.nslab + s) * q_slab_bytes,
+                                              &tmQ, &sm.bar[kBarQFull + qb], s * 64, 0, h * g.G,
+                                              bb, l, keep);
+                    qb ^= 1;
+                    if (qb == 0)
+                        qph ^= 1;
+                    const uint64_t pol = T.phase == 2 ? drop : keep;
+                    for (int tile = 0; tile < T.ntiles; ++tile) {
+                        c0 = clock64();
+                        if (!wait_bar(&sm.bar[kBarKEmpty + ks], kph ^ 1, flag, a)) {
+                            ok = false;
+                            break;
+                        }
+                        cy_wk += clock64() - c0;
+                        ptx::mbar_arrive_expect_tx(&sm.bar[kBarKFull + ks],
+                                                   (uint32_t)a.nslab * kSlabBytes);
+                        flag[kFlagKArm + ks] = (int)kph;
+                        for (int s = 0; s < a.nslab; ++s)
+                            ptx::tma_load_5d_hint(sm.k + ((size_t)ks * a.nslab + s) * kSlabBytes,
+                                                  &tmK, &sm.bar[kBarKFull + ks], s * 64,
+                                                  T.k_lo + tile * kTile, h, bb, l, pol);
+                        if (++ks == a.kstages) {
+                            ks = 0;
+                            kph ^= 1;
+                        }
+                    }
+                }
+            trace_put(a, kTrProdWaitQ, cy_wq);
+            trace_put(a, kTrProdWaitK, cy_wk);
+            trace_put(a, kTrProdTotal, clock64() - cy0);
+        }
+    } else if (warp == 1) {
+        // ---- MMA issuer -----------------------------------------------------------------
+        if (lane == 0) {
+            const uint32_t idesc = ptx::idesc_bf16_f32(kTile, a.r_pad);
+            int ks = 0, qb = 0;
+            uint32_t kph = 0, qph = 0;
+            int64_t tc = 0;  // accumulator sequence number: buffer tc % 3, use tc / 3
+            long long cy_wq = 0, cy_wk = 0, cy_wa = 0, cy_is = 0, cy_cm = 0;
+            const long long cy0 = clock64();
+            bool ok = true;
+            for (int64_t t = 0; ok && t <= a.steps; ++t)
+                for (int j = 0; ok && j < 2; ++j) {
+                    Task T;
+                    if (!get_task(a, t, j, T))
+                        continue;
+                    long long c0 = clock64();
+                    if (!wait_bar(&sm.bar[kBarQFull + qb], qph, flag, a)) {
+                        ok = false;
+                        break;
+                    }
+                    cy_wq += clock64() - c0;
+                    const uint32_t qbase = ptx::smem_addr(sm.q + (size_t)qb * a.nslab * q_slab_bytes);
+                    for (int tile = 0; tile < T.ntiles; ++tile, ++tc) {
+                        const int ab = (int)(tc % kAccBufs);
+                        const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
+                        c0 = clock64();
+                        if (!wait_bar(&sm.bar[kBarKFull + ks], kph, flag, a)) {
+                            ok = false;
+                            break;
+                        }
+                        long long c1 = clock64();
+                        cy_wk += c1 - c0;
+                        if (!wait_bar(&sm.bar[kBarAccEmpty + ab], aph ^ 1, flag, a)) {
+                            ok = false;
+                            break;
+                        }
+                        c0 = clock64();
+                        cy_wa += c0 - c1;
+                        ptx::tc_fence_after();
+                        // Descriptors are linear in the start address (bits 0..13 hold
+                        // addr >> 4), so each K step adds its byte offset / 16.
+                        const uint64_t ad0 = ptx::smem_desc_sw128(
+                            ptx::smem_addr(sm.k + (size_t)ks * a.nslab * kSlabBytes));
+                        const uint64_t bd0 = ptx::smem_desc_sw128(qbase);
+                        const uint32_t d_tmem = tmem_base + (uint32_t)(ab * a.acc_stride);
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            if (kk < a.nslab * 4) {
+                                const uint32_t a_off = ((uint32_t)(kk >> 2) * kSlabBytes +
+                                                        (uint32_t)(kk & 3) * 32u) >> 4;
+                                const uint32_t b_off = ((uint32_t)(kk >> 2) * q_slab_bytes +
+                                                        (uint32_t)(kk & 3) * 32u) >> 4;
+                                ptx::mma_bf16(d_tmem, ad0 + a_off, bd0 + b_off, idesc,
+                                              kk > 0 ? 1u : 0u);
+                            }
+                        }
+                        c1 = clock64();
+                        cy_is += c1 - c0;
+                        ptx::mma_commit(&sm.bar[kBarKEmpty + ks]);
+                        ptx::mma_commit(&sm.bar[kBarAccFull + ab]);
+                        cy_cm += clock64() - c1;
+                        if (++ks == a.kstages) {
+                            ks = 0;
+                            kph ^= 1;
+                        }
+                    }
+                    if (!ok)
+                        break;
+                    ptx::mma_commit(&sm.bar[kBarQEmpty + qb]);
+                    qb ^= 1;
+                    if (qb == 0)
+                        qph ^= 1;
+                }
+            trace_put(a, kTrMmaWaitQ, cy_wq);
+            trace_put(a, kTrMmaWaitK, cy_wk);
+            trace_put(a, kTrMmaWaitAcc, cy_wa);
+            trace_put(a, kTrMmaIssue, cy_is);
+            trace_put(a, kTrMmaCommit, cy_cm);
+            trace_put(a, kTrMmaTotal, clock64() - cy0);
+            trace_put(a, kTrTiles, tc);
+            // Every MMA issued so far completes before the drain barrier fires.
+            ptx::mma_commit(&sm.bar[kBarDrain]);
+            drain_bar(&sm.bar[kBarDrain], 0, 2000000000ull);
+        }
+    } else {
+        // ---- coordinator (warps 2, 3) ----------------------------------------------------
+        // Per step: (a) for the coming phase-2 task, wait until every chunk of its unit has
+        // reported (the unit counter), merge the chunk sums into -lse and hand them to the
+        // epilogue; (b) for the phase-1 task the epilogue is finishing, add its per-warp row
+        // sums, publish them to global memory and count the chunk in.
+        const int ct = threadIdx.x - 64;  // 0 .. kCoordThreads-1
+        bool dead = false;
+        auto wait_c = [&](uint64_t *bar, uint32_t parity) {
+            if (!dead) {
+                const bool got = wait_bar(bar, parity, flag, a);
+                dead = !__all_sync(0xffffffffu, got);
+            }
+            return !dead;
+        };
+        int p1c = 0, p2c = 0;
+        for (int t = 0; t <= (int)a.steps; ++t) {
+            Task T;
+            if (get_task(a, t, 1, T)) {
+                const int lb = p2c & 1;
+                const uint32_t lph = (uint32_t)((p2c >> 1) & 1);
+                ++p2c;
+                // Every named barrier below is reached by both warps on every path.
+                const bool ok = wait_c(&sm.bar[kBarLseEmpty + lb], lph ^ 1);
+                if (ct == 0 && ok) {
+                    // Every chunk of the unit has published its row sums.
+                    const uint64_t t0 = ptx::globaltimer();
+                    while (ptx::ld_acquire_u32(&a.count[T.u]) < (uint32_t)a.nchunks) {
+                        __nanosleep(64);
+                        if (flag[kFlagAbort] || *(volatile uint32_t *)a.status != 0) {
+                            flag[kFlagAbort] = 1;
+                            break;
+                        }
+                        if (ptx::globaltimer() - t0 > a.timeout_ns) {
+                            flag[kFlagAbort] = 1;
+                            set_status(a.status, DGE_ERR_DEVICE_TIMEOUT);
+                            break;
+                        }
+                    }
+                }
+                ptx::named_barrier(kBarCoord, kCoordThreads);
+                if (ok) {
+                    float *L = sm.sL + lb * 256;
+                    for (int r = ct; r < a.r_pad; r += kCoordThreads) {
+                        float v = -INFINITY;
+                        if (r < g.R) {
+                            float Z = 0.f;
+                            for (int c = 0; c < a.nchunks; ++c)
+                                Z += __ldcg(&a.part[(T.u * a.nchunks + c) * g.R + r]);
+                            if (!(Z >= 0x1p-60f && Z < 0x1p126f))
+                                flag[kFlagBad] = 1;
+                            v = -log2f(Z);
+                        }
+                        L[r] = v;
+                    }
+                }
+                ptx::named_barrier(kBarCoord, kCoordThreads);
+                const int bad = flag[kFlagBad];
+                ptx::named_barrier(kBarCoord, kCoordThreads);
+                if (ct == 0) {
+                    sm.sLbad[lb] = (bad || flag[kFlagAbort] || !ok) ? 1 : 0;
+                    if (bad)
+                        a.ready[T.u] = kReadyBad;  // recomputed after the kernel
+                    flag[kFlagBad] = 0;
+                    ptx::mbar_arrive(&sm.bar[kBarLseFull + lb]);
+                }
+            }
+            if (get_task(a, t, 0, T)) {
+                const int rb = p1c & 1;
+                const uint32_t rph = (uint32_t)((p1c >> 1) & 1);
+                ++p1c;
+                const bool ok = wait_c(&sm.bar[kBarRedFull + rb], rph);
+                if (ok) {
+                    constexpr int W = kMaxGroups * 16;
+                    for (int col = ct; col < g.R; col += kCoordThreads) {
+                        int w = 0;
+                        while (w + 1 < kEpiWG && col >= a.gbase[w + 1] * 16)
+                            ++w;
+                        const int lc = col - a.gbase[w] * 16;
+                        const float *rbuf = sm.red + (rb * kEpiWG + w) * 4 * W;
+                        const float sum = rbuf[lc] + rbuf[W + lc] + rbuf[2 * W + lc] + rbuf[3 * W + lc];
+                        a.part[(T.u * a.nchunks + T.chunk) * g.R + col] = sum;
+                    }
+                }
+                ptx::named_barrier(kBarCoord, kCoordThreads);
+                if (ct == 0) {
+                    if (ok) {
+                        // The barrier orders every row-sum store before this cumulative
+                        // release of the chunk count.
+                        ptx::fence_acq_rel_gpu();
+                        atomicAdd(&a.count[T.u], 1u);
+                    }
+                    ptx::mbar_arrive(&sm.bar[kBarRedEmpty + rb]);
+                }
+            }
+        }
+    }
+    } else {
+        ptx::regs_inc<kRegsEpilogue>();
+        // ---- epilogue -------------------------------------------------------------------
+        // Every warpgroup reads every tile, its own 16-column groups: phase 1 keeps row sums
+        // in registers, phase 2 forms partial column sums that warpgroup 0 collects.
+        const int ew = warp - kEpiWarp0;         // 0 .. kEpiWarps-1
+        const int wg = ew >> 2;                  // warpgroup
+        const int quarter = warp & 3;            // TMEM lane quarter of this warp
+        const int kl = quarter * 32 + lane;      // key within the tile
+        const int wi = (ew & 3) * 32 + lane;     // thread index within the warpgroup
+        const int ng = a.ng[wg];
+        const int col_base = a.gbase[wg] * 16;
+        const int ngroups = a.r_pad / 16;
+        const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+        const float s2 = g.scale_log2;
+        const int first_causal = g.n - g.m;      // keys from here on are not seen by every row
+        int tc = 0;   // accumulator tiles consumed (buffer tc % 3, use tc / 3)
+        int xc = 0;   // phase-2 tiles (exchange buffer xc % 2, use xc / 2)
+        int p1c = 0;  // phase-1 tasks (row-sum hand-off buffer p1c % 2)
+        int p2c = 0;  // phase-2 tasks (-lse buffer p2c % 2)
+        bool dead = false;
+
+        long long cy_wa = 0, cy_x = 0, cy_p1e = 0, cy_p2s = 0;
+        const long long cy0 = clock64();
+        // Waits for this thread's accumulator and returns false once the CTA is dead
+        // (the outcome is warp-uniform: the TMEM loads after it are warp-collective).
+        auto acquire_acc = [&](int ab, uint32_t aph) {
+            const long long c0 = clock64();
+            if (!dead) {
+                const bool got = wait_bar(&sm.bar[kBarAccFull + ab], aph, flag, a);
+                dead = !__all_sync(0xffffffffu, got);
+            }
+            if (!dead)
+                ptx::tc_fence_after();
+            cy_wa += clock64() - c0;
+            return !dead;
+        };
+        // A bounded, warp-uniform wait on a CTA barrier (false once the CTA is dead).
+        auto wait_uniform = [&](uint64_t *bar, uint32_t parity) {
+            const long long c0 = clock64();
+            if (!dead) {
+                const bool got = wait_bar(bar, parity, flag, a);
+                dead = !__all_sync(0xffffffffu, got);
+            }
+            cy_x += clock64() - c0;
+            return !dead;
+        };
+        auto release_acc = [&](int ab, uint32_t count) {
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0 && !dead)
+                ptx::mbar_arrive_cnt(&sm.bar[kBarAccEmpty + ab], count);
+        };
+
+        for (int t = 0; t <= (int)a.steps; ++t)
+            for (int j = 0; j < 2; ++j) {
+                Task T;
+                if (!get_task(a, t, j, T))
+                    continue;
+                if (T.phase == 1) {
+                    // ---------------- phase 1: row sums over this chunk ----------------
+                    float z[kMaxGroups][16];
+#pragma unroll
+                    for (int i = 0; i < kMaxGroups; ++i)
+#pragma unroll
+                        for (int c = 0; c < 16; ++c)
+                            z[i][c] = 0.f;
+                    for (int tile = 0; tile < T.ntiles; ++tile, ++tc) {
+                        const int ab = tc % kAccBufs;
+                        const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
+                        const int tile0 = T.k_lo + tile * kTile;
+                        const int key = tile0 + kl;
+                        const bool valid = key < T.k_hi;
+                        const bool causal = tile0 + kTile > first_causal;
+                        if (acquire_acc(ab, aph)) {
+                            // One 16-column group per TMEM round trip (a few tens of cycles).
+                            const uint32_t tbase =
+                                tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
+#pragma unroll
+                            for (int gi = 0; gi < kMaxGroups; ++gi)
+                                if (gi < ng) {
+                                    float v[16];
+                                    ptx::tmem_ld16(tbase + gi * 16, v);
+                                    ptx::tmem_ld_wait();
+                                    rows_add(z[gi], v, s2, valid, causal, key, first_causal,
+                                             col_base + gi * 16, g.m);
+                                }
+                        }
+                        release_acc(ab, 1u);
+                    }
+                    const long long c_end = clock64();
+                    // Sums over this warp's 32 keys, handed to the coordinator warps through
+                    // a double-buffered area (they add the warps in a fixed order).
+                    const int rb = p1c & 1;
+                    const uint32_t rph = (uint32_t)((p1c >> 1) & 1);
+#pragma unroll
+                    for (int gi = 0; gi < kMaxGroups; gi += 2) {
+                        if (gi < ng) {
+                            if (gi + 1 < kMaxGroups && gi + 1 < ng)
+                                transpose_sum32(z[gi], z[gi + 1 < kMaxGroups ? gi + 1 : gi], lane);
+                            else
+                                transpose_sum16(z[gi], lane);
+                        }
+                    }
+                    if (wait_uniform(&sm.bar[kBarRedEmpty + rb], rph ^ 1)) {
+                        float *red = sm.red + ((rb * kEpiWG + wg) * 4 + quarter) * (kMaxGroups * 16);
+#pragma unroll
+                        for (int gi = 0; gi < kMaxGroups; gi += 2) {
+                            if (gi < ng) {
+                                if (gi + 1 < kMaxGroups && gi + 1 < ng)
+                                    red[gi * 16 + lane] = z[gi][0];
+                                else if (lane < 16)
+                                    red[gi * 16 + lane] = z[gi][0];
+                            }
+                        }
+                        __syncwarp();
+                        if (lane == 0)
+                            ptx::mbar_arrive(&sm.bar[kBarRedFull + rb]);
+                    }
+                    ++p1c;
+                    cy_p1e += clock64() - c_end;
+                } else {
+                    const long long c_start = clock64();
+                    // ---------------- phase 2: column sums of this chunk ----------------
+                    // The coordinator warps have put -lse of this unit's rows in sL[lb].
+                    const int lb = p2c & 1;
+                    const uint32_t lph = (uint32_t)((p2c >> 1) & 1);
+                    float nL[kMaxGroups][16];
+                    bool task_ok = false;
+                    if (wait_uniform(&sm.bar[kBarLseFull + lb], lph)) {
+                        const float *L = sm.sL + lb * 256 + col_base;
+#pragma unroll
+                        for (int gi = 0; gi < kMaxGroups; ++gi)
+#pragma unroll
+                            for (int c = 0; c < 16; ++c)
+                                nL[gi][c] = gi < ng ? L[gi * 16 + c] : -INFINITY;
+                        task_ok = sm.sLbad[lb] == 0;
+                        __syncwarp();
+                        if (lane == 0)
+                            ptx::mbar_arrive(&sm.bar[kBarLseEmpty + lb]);
+                    } else {
+#pragma unroll
+                        for (int gi = 0; gi < kMaxGroups; ++gi)
+#pragma unroll
+                            for (int c = 0; c < 16; ++c)
+                                nL[gi][c] = -INFINITY;
+                    }
+                    task_ok = task_ok && !dead;
+                    ++p2c;
+                    cy_p2s += clock64() - c_start;
+                    for (int tile = 0; tile < T.ntiles; ++tile, ++tc, ++xc) {
+                        const int ab = tc % kAccBufs;
+                        const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
+                        const int tile0 = T.k_lo + tile * kTile;
+                        const int key = tile0 + kl;
+                        const bool causal = tile0 + kTile > first_causal;
+                        float2 acc = make_float2(0.f, 0.f);
+                        if (acquire_acc(ab, aph)) {
+                            const uint32_t tbase =
+                                tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
+#pragma unroll
+                            for (int gi = 0; gi < kMaxGroups; ++gi)
+                                if (gi < ng) {
+                                    float v[16];
+                                    ptx::tmem_ld16(tbase + gi * 16, v);
+                                    ptx::tmem_ld_wait();
+                                    col_add(acc, v, nL[gi], s2, causal, key, first_causal,
+                                            col_base + gi * 16, g.m);
+                                }
+                        }
+                        release_acc(ab, 1u);
+                        // Warpgroups 1.. hand their partial sums to warpgroup 0 through a
+                        // double-buffered exchange; warpgroup 0 adds them in a fixed order.
+                        const int xb = xc & 1;
+                        const uint32_t xph = (uint32_t)((xc >> 1) & 1);
+                        float *xrow = sm.xch + xb * (kEpiWG - 1) * kTile;
+                        if (wg > 0) {
+                            if (wait_uniform(&sm.bar[kBarXEmpty + xb], xph ^ 1)) {
+                                xrow[(wg - 1) * kTile + kl] = acc.x + acc.y;
+                                __syncwarp();
+                                if (lane == 0)
+                                    ptx::mbar_arrive(&sm.bar[kBarXFull + xb]);
+                            }
+                        } else {
+                            if (wait_uniform(&sm.bar[kBarXFull + xb], xph)) {
+                                float total = acc.x + acc.y;
+#pragma unroll
+                                for (int w = 0; w < kEpiWG - 1; ++w)
+                                    total += xrow[w * kTile + kl];
+                                if (task_ok && key < T.k_hi)
+                                    a.raw[T.u * g.P + key] = total;
+                                __syncwarp();
+                                if (lane == 0)
+                                    ptx::mbar_arrive(&sm.bar[kBarXEmpty + xb]);
+                            }
+                        }
+                    }
+                }
+            }
+        if (ew == 0 && lane == 0) {
+            trace_put(a, kTrEpiWaitAcc, cy_wa);
+            trace_put(a, kTrEpiExchange, cy_x);
+            trace_put(a, kTrEpiP1End, cy_p1e);
+            trace_put(a, kTrEpiP2Start, cy_p2s);
+            trace_put(a, kTrEpiTotal, clock64() - cy0);
+        }
+    }
+
+    // ---- teardown ------------------------------------------------------------------------
+    __syncthreads();
+    if (warp == 0 && lane == 0) {
+        // Copies still in flight (only after an abort) land before the CTA leaves.
+        for (int i = 0; i < a.kstages; ++i)
+            if (flag[kFlagKArm + i] >= 0)
+                drain_bar(&sm.bar[kBarKFull + i], (uint32_t)flag[kFlagKArm + i], 1000000000ull);
+        for (int i = 0; i < 2; ++i)
+            if (flag[kFlagQArm + i] >= 0)
+                drain_bar(&sm.bar[kBarQFull + i], (uint32_t)flag[kFlagQArm + i], 1000000000ull);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 1)
+        ptx::tmem_dealloc(tmem_base, kTmemCols);
+}
+
+using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                            const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                            const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                            CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+Encode encode_fn()
+{
+    static Encode fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<Encode>(p);
+    }
+    return fn;
+}
+
+// 5-D map over [L][b][heads][rows][d] with box {64, box_rows, box_heads, 1, 1}.
+bool encode_5d(CUtensorMap *map, const TensorDesc &t, int L, int b, int heads, int rows, int d,
+               int box_rows, int box_heads)
+{
+    Encode fn = encode_fn();
+    if (!fn)
+        return false;
+    const cuuint64_t dims[5] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)heads, (cuuint64_t)b,
+                                (cuuint64_t)L};
+    const cuuint64_t strides[4] = {(cuuint64_t)t.s_pos * 2, (cuuint64_t)t.s_head * 2,
+                                   (cuuint64_t)t.s_batch * 2, (cuuint64_t)t.s_layer * 2};
+    const cuuint32_t box[5] = {64, (cuuint32_t)box_rows, (cuuint32_t)box_heads, 1, 1};
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    for (int i = 0; i < 4; ++i)
+        if (strides[i] == 0 || strides[i] % 16 != 0)
+            return false;
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<__nv_bfloat16 *>(t.data), dims,
+              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+unsigned long long *g_trace = nullptr;
+int g_trace_cta = 0;
+
+}  // namespace
+
+void tc_set_trace(unsigned long long *buffer, int cta)
+{
+    g_trace = buffer;
+    g_trace_cta = cta;
+}
+
+bool tc_supported(const Geometry &g)
+{
+    if (g.variant != DGE_VARIANT_SCORED || (g.d != 64 && g.d != 128) ||
+        g.R > kEpiWG * kMaxGroups * 16 || g.m > 256 || g.G > 256)
+        return false;
+    int dev = 0, major = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess)
+        return false;
+    return major == 10 && encode_fn() != nullptr;
+}
+
+TcPlan tc_plan(const Geometry &g)
+{
+    TcPlan p;
+    p.r_pad = (g.R + 15) & ~15;
+    p.nslab = g.d / 64;
+    p.chunk_keys = 1024;
+    p.nchunks = (g.n + p.chunk_keys - 1) / p.chunk_keys;
+    p.kstages = kMaxKStages;
+    while (p.kstages > 2 && smem_bytes(p.r_pad, p.nslab, p.kstages) > 232448)
+        --p.kstages;
+    p.smem = smem_bytes(p.r_pad, p.nslab, p.kstages);
+    // At least half of the SM's shared memory: one CTA per SM, so a CTA's TMEM allocation
+    // (all 512 columns) never waits for another CTA of this kernel.
+    if (p.smem < 120 * 1024)
+        p.smem = 120 * 1024;
+    return p;
+}
+
+cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                            const TcPlan &plan, const TcBuffers &buf, cudaStream_t stream,
+                            bool *encoded)
+{
+    CUtensorMap tmK, tmQ;
+    *encoded = encode_5d(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d, kTile, 1) &&
+               encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.m, g.d, g.m, g.G);
+    if (!*encoded)
+        return cudaSuccess;
+    int dev = 0, sms = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err == cudaSuccess)
+        err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess)
+        return err;
+
+    TcArgs a;
+    a.g = g;
+    a.r_pad = plan.r_pad;
+    a.acc_stride = (plan.r_pad + 31) & ~31;
+    a.nslab = plan.nslab;
+    a.kstages = plan.kstages;
+    a.chunk_keys = plan.chunk_keys;
+    a.nchunks = plan.nchunks;
+    a.items = g.U * plan.nchunks;
+    const int NG = plan.r_pad / 16;
+    for (int w = 0, base = 0; w < kEpiWG; ++w) {
+        a.ng[w] = NG / kEpiWG + (w < NG % kEpiWG ? 1 : 0);
+        a.gbase[w] = base;
+        base += a.ng[w];
+    }
+    const int64_t grid = a.items < sms ? a.items : sms;
+    a.steps = (a.items + grid - 1) / grid;
+    a.part = buf.part;
+    a.lse2 = buf.lse2;
+    a.raw = buf.raw;
+    a.count = buf.count;
+    a.ready = buf.ready;
+    a.status = buf.status;
+    a.timeout_ns = 4000000000ull;
+    a.trace = g_trace;
+    a.trace_cta = g_trace_cta;
+
+    void (*kernel)(const CUtensorMap, const CUtensorMap, const TcArgs) = score_tc_kernel;
+    err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)plan.smem);
+    if (err != cudaSuccess)
+        return err;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = plan.smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, tmK, tmQ, a);
+}
+
+}  // namespace dge

@@ -192,3 +192,85 @@ def test_full_size_sampled_units(name):
             assert np.all(blk[:, -wl.tail:] == np.arange(wl.n - wl.tail, wl.n))
     del tens, out
     torch.cuda.empty_cache()
+
+
+# --- the two scoring kernel families ----------------------------------------------------
+
+@pytest.fixture
+def mma_path(monkeypatch):
+    """Force the warp-level (mma.sync) scoring kernels for the duration of a test."""
+    monkeypatch.setenv("DGE_SCORE_KERNEL", "mma")
+    yield
+
+
+@pytest.mark.parametrize("name", ["c2_small", "c3_small", "gqa8_ragged", "short_cache"])
+def test_warp_level_path_matches_oracle(mma_path, name):
+    wl = SMALL[name]
+    tens, out = run(wl)
+    check_all(wl, tens, out)
+
+
+def _kernels_run(fn):
+    from paper_2609_33334_gb300 import binding as B
+    B.dge_profile_begin()
+    fn()
+    torch.cuda.synchronize()
+    return {name for name, _, _ in B.dge_profile_end()}
+
+
+@pytest.mark.parametrize("name,expect_tc", [("c2_small", True), ("c1_tiny", True),
+                                            ("c5_small", False), ("c4_small", False)])
+def test_tensor_core_path_is_taken_where_eligible(name, expect_tc):
+    wl = SMALL.get(name) or WL[name]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    names = _kernels_run(lambda: api.evict(p, tens["K"], tens["V"], tens["Q"]))
+    assert ("score_tc" in names) == expect_tc, names
+
+
+def test_paths_agree_closely():
+    """tcgen05 and mma.sync scores agree far inside the oracle tolerance."""
+    import os
+    wl = SMALL["c3_small"]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    a = api.score(p, tens["K"], tens["Q"])
+    os.environ["DGE_SCORE_KERNEL"] = "mma"
+    try:
+        b = api.score(p, tens["K"], tens["Q"])
+    finally:
+        del os.environ["DGE_SCORE_KERNEL"]
+    torch.cuda.synchronize()
+    rel = ((a - b).abs() / b.abs().clamp_min(1e-30)).max().item()
+    assert rel < 1e-4, rel
+
+
+def test_large_logits_are_recomputed_exactly():
+    """Logits far beyond fp32's unshifted exponent range take the recompute path."""
+    wl = WL["c1_tiny"].with_(L=1, budgets=(128,))
+    tens = inputs.make_inputs(wl, device="cuda")
+    tens["Q"] = (tens["Q"].float() * 24.0).to(torch.bfloat16)   # logits ~ 100+ nats
+    tens, out = run(wl, tens=tens)
+    check_all(wl, tens, out)
+
+
+def test_tail_shorter_than_observation_rows():
+    """tail < m: observation rows see only their causal prefix of the scored range."""
+    wl = WL["c1_tiny"].with_(n=700, n_spans=0)
+    tens = inputs.make_inputs(wl, device="cuda")
+    tail = 3
+    p = api.problem_from_workload(wl)
+    p.tail = tail
+    out = api.evict(p, tens["K"], tens["V"], tens["Q"], want_scores=True)
+    torch.cuda.synchronize()
+    for h in range(wl.Hkv):
+        Qg = inputs.bf16_bits(tens["Q"][0, 0, h * wl.G:(h + 1) * wl.G])
+        ref = oracle.evict_unit(Qg, inputs.bf16_bits(tens["K"][0, 0, h]),
+                                inputs.bf16_bits(tens["V"][0, 0, h]), variant=0, m=wl.m,
+                                tail=tail, sinks=0, budget=wl.budgets[0], pool_kind=wl.pool,
+                                kernel=wl.pool_kernel)
+        from parity import assert_scores_close, check_kept
+        assert_scores_close(out["scores"][h].cpu().numpy(), ref["pooled"])
+        r0 = h * wl.budgets[0]
+        check_kept(out["idx"][r0:r0 + wl.budgets[0]].cpu().numpy(), ref["pooled"], ref["idx"],
+                   n=wl.n, sinks=0, tail=tail, budget=wl.budgets[0])
