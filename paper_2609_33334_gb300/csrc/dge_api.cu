@@ -220,7 +220,7 @@ int make_plan(const dge_problem *p, Plan &plan)
         size_t part_bytes = (size_t)g.U * g.R * plan.nchunks * sizeof(float2);
         if (p->variant == DGE_VARIANT_SCORED) {
             plan.tc = tc_plan(g);
-            const size_t tc_bytes = (size_t)g.U * g.R * plan.tc.nchunks * sizeof(float);
+            const size_t tc_bytes = (size_t)g.U * plan.tc.r4 * plan.tc.nchunks * sizeof(float);
             if (tc_bytes > part_bytes)
                 part_bytes = tc_bytes;
         }

@@ -21,10 +21,11 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
 // Scoring on the tcgen05 path (score_tc.cu).
 struct TcPlan {
     int r_pad, nslab, chunk_keys, nchunks, kstages;
+    int r4;            // row stride of the chunk sums: R rounded up to 4 (16-byte rows)
     size_t smem;
 };
 struct TcBuffers {
-    float *part;       // [U][nchunks][R] row sums of each key chunk
+    float *part;       // [U][nchunks][r4] row sums of each key chunk
     float *lse2;       // [U][R]
     float *raw;        // [U][P]
     uint32_t *count;   // [U], zero before the launch

@@ -8,17 +8,20 @@
 //   warp 0      TMA producer: the unit's stacked query block (5-D box, G heads x m
 //               rows) and 128-key tiles of K, 128-byte swizzled, into a ring;
 //   warp 1      MMA issuer: D[128 keys x R_pad rows] = K_tile . Q^T with
-//               tcgen05.mma (M = 128, N = R_pad <= 256, bf16 -> fp32) into one of
-//               two TMEM accumulators; also owns the TMEM allocation;
-//   warps 2-9   epilogue: two warpgroups, each thread one key (TMEM lane), each
-//               warpgroup half of the row columns.
+//               tcgen05.mma (M = 128, N = R_pad, bf16 -> fp32) into one of three
+//               TMEM accumulators; also owns the TMEM allocation;
+//   warps 2-3   coordinator: warp 3 publishes the phase-1 chunk sums and counts
+//               them into the unit; warp 2 merges a finished unit's chunk sums
+//               (bulk-copied to shared memory) into -lse for this CTA's phase-2
+//               tasks;
+//   warps 4-15  epilogue: three warpgroups, each thread one key (TMEM lane),
+//               each warpgroup a third of the row columns.
 // Work items are (unit, key chunk).  Step t of CTA s runs phase 1 of item
-// t*S + s (per-row sums 2^x over the chunk, reduced across the 128 keys at the
-// end) and then phase 2 of item (t-1)*S + s (2^{x - lse} summed over rows per
-// key), so phase 2 re-reads a chunk this CTA streamed one step earlier, from L2.
-// The last phase-1 task of a unit merges the chunk sums into lse and publishes
-// a ready flag; phase-2 tasks wait for it (bounded).  Row sums use no running
-// maximum: fp32 holds 2^x for |x| < 126, and a unit whose sums leave
+// t*S + s (per-row sums 2^x over the chunk) and then phase 2 of item
+// (t-1)*S + s - (nchunks-1) (2^{x - lse} summed over rows per key), so phase 2
+// re-reads a chunk streamed about one step earlier while it is still in L2, and
+// only needs units whose every chunk finished phase 1 in an earlier step.  Row sums use no
+// running maximum: fp32 holds 2^x for |x| < 126, and a unit whose sums leave
 // [2^-60, 2^126) is flagged (ready = 2) and recomputed by the warp-level path.
 //
 // Every wait is bounded: on expiry the CTA records DGE_ERR_DEVICE_TIMEOUT in the
@@ -47,34 +50,34 @@ constexpr int kRegsLaunch = 128, kRegsControl = 56, kRegsEpilogue = 152;
 static_assert(4 * 32 * kRegsControl + kEpiWarps * 32 * kRegsEpilogue <= kThreads * kRegsLaunch,
               "register split");
 constexpr int kMaxGroups = 3;             // 16-column groups per epilogue warpgroup
-constexpr int kBarAllEpi = 1 + kEpiWG;    // named barrier of all epilogue warps (1..: one per WG)
 constexpr int kMaxKStages = 4;
 constexpr int kAccBufs = 3;               // TMEM accumulators
 constexpr int kTmemCols = 512;
 constexpr int kSlabBytes = kTile * 128;  // 128 rows x 64 bf16
-constexpr uint32_t kReadyOk = 1, kReadyBad = 2;
+constexpr uint32_t kReadyBad = 2;          // unit left fp32's range: recomputed afterwards
 
 // Barrier slots.
 constexpr int kBarKFull = 0, kBarKEmpty = 4, kBarQFull = 8, kBarQEmpty = 10, kBarAccFull = 12,
-              kBarAccEmpty = 15, kBarDrain = 18, kBarXFull = 19, kBarXEmpty = 21, kBarRedFull = 23,
-              kBarRedEmpty = 25, kBarLseFull = 27, kBarLseEmpty = 29, kNumBars = 31;
-constexpr int kBarCoord = 1 + kEpiWG + 1;  // named barrier of the two coordinator warps
-constexpr int kCoordThreads = 64;          // warps 2 and 3
-// Flag slots (ints): abort, last-arrival, wait result, out-of-range, then the parity of
-// the last arm of every key stage and query buffer (-1 = never armed) for the drain.
-constexpr int kFlagAbort = 0, kFlagLast = 1, kFlagWait = 2, kFlagBad = 3, kFlagKArm = 4,
-              kFlagQArm = 8;
+              kBarAccEmpty = 15, kBarDrain = 18, kBarRedFull = 19, kBarRedEmpty = 21,
+              kBarLseFull = 23, kBarLseEmpty = 25, kBarStage = 27, kNumBars = 28;
+constexpr int kStageBytes = 12288;        // chunk sums of a unit, staged for the lse merge
+constexpr int kCtrlBytes = 320;            // barriers, TMEM address, flags (16-byte multiple)
+constexpr int kRowsPerLane = 5;           // rows of the lse merge per lane (R <= 160)
+// Flag slots (ints): abort, then the parity of the last arm of every key stage, query
+// buffer and the staging buffer (-1 = never armed) for the drain.
+constexpr int kFlagAbort = 0, kFlagKArm = 4, kFlagQArm = 8, kFlagSArm = 10;
 
 struct TcArgs {
     Geometry g;
-    int r_pad, nslab, kstages;
+    int r_pad, r4, nslab, kstages;
     int acc_stride;    // TMEM columns between accumulator buffers
     int chunk_keys, nchunks;
     int64_t items;
+    int64_t lag;       // extra items between an item's phase-1 and phase-2 tasks
     int ng[kEpiWG];    // 16-column groups of each epilogue warpgroup
     int gbase[kEpiWG]; // first group of each epilogue warpgroup
     int64_t steps;
-    float *part;       // [U][nchunks][R]
+    float *part;       // [U][nchunks][r4]
     float *lse2;       // [U][R]
     float *raw;        // [U][P]
     uint32_t *count;   // [U]
@@ -89,14 +92,29 @@ struct TcArgs {
 // CTA at the end into trace[slot * DGE_TRACE_LEN + blockIdx.x].
 enum TraceSlot {
     kTrMmaWaitQ = 0, kTrMmaWaitK, kTrMmaWaitAcc, kTrMmaIssue, kTrMmaCommit, kTrMmaTotal,
-    kTrProdWaitQ, kTrProdWaitK, kTrProdTotal, kTrEpiWaitAcc, kTrEpiTiles, kTrEpiP1End,
-    kTrEpiP2Start, kTrEpiExchange, kTrEpiTotal, kTrTiles
+    kTrProdWaitQ, kTrProdWaitK, kTrProdTotal, kTrEpiWaitAcc, kTrStepTimeline, kTrEpiP1End,
+    kTrEpiP2Start, kTrTimeline, kTrEpiTotal, kTrTiles
 };
 
 __device__ __forceinline__ void trace_put(const TcArgs &a, int slot, long long v)
 {
     if (a.trace && blockIdx.x < DGE_TRACE_LEN)
         a.trace[slot * DGE_TRACE_LEN + blockIdx.x] = (unsigned long long)v;
+}
+
+// Timeline of CTA a.trace_cta: global-timer stamps (ns) at index i of a timeline slot.
+__device__ __forceinline__ void trace_at(const TcArgs &a, int slot, int i)
+{
+    if (a.trace && (int)blockIdx.x == a.trace_cta && i >= 0 && i < DGE_TRACE_LEN)
+        a.trace[slot * DGE_TRACE_LEN + i] = ptx::globaltimer();
+}
+
+// Step timeline of every CTA: global-timer stamp of its phase-1 task i at i * grid + cta.
+__device__ __forceinline__ void trace_step(const TcArgs &a, int slot, int i)
+{
+    const int64_t idx = (int64_t)i * gridDim.x + blockIdx.x;
+    if (a.trace && idx < DGE_TRACE_LEN)
+        a.trace[slot * DGE_TRACE_LEN + idx] = ptx::globaltimer();
 }
 
 struct Task {
@@ -106,7 +124,9 @@ struct Task {
 };
 
 // Task j (0: phase 1, 1: phase 2) of step t for this CTA: phase 1 of item t*S + s, phase 2
-// of item (t-1)*S + s.  False when there is none (or it covers no keys).
+// of item (t-1)*S + s - lag.  With lag = nchunks - 1, every unit a phase-2 task needs was
+// completed by phase-1 tasks of earlier steps (a unit's chunks may straddle two steps).
+// False when there is none (or it covers no keys).
 __device__ __forceinline__ bool get_task(const TcArgs &a, int64_t t, int j, Task &T)
 {
     const int64_t S = gridDim.x, s = blockIdx.x;
@@ -115,12 +135,10 @@ __device__ __forceinline__ bool get_task(const TcArgs &a, int64_t t, int j, Task
         item = t * S + s;
         T.phase = 1;
     } else {
-        if (t < 1)
-            return false;
-        item = (t - 1) * S + s;
+        item = (t - 1) * S + s - a.lag;
         T.phase = 2;
     }
-    if (item >= a.items)
+    if (item < 0 || item >= a.items)
         return false;
     T.u = item / a.nchunks;
     T.chunk = (int)(item % a.nchunks);
@@ -136,13 +154,15 @@ __device__ __forceinline__ bool get_task(const TcArgs &a, int64_t t, int j, Task
 struct Smem {
     uint8_t *q;          // [2][nslab][r_pad * 128]
     uint8_t *k;          // [kstages][nslab][kSlabBytes]
+    float *stage;        // [kStageBytes / 4] chunk sums of one unit (lse merge)
     uint64_t *bar;       // [kNumBars]
     uint32_t *tmem;      // allocation result
     int *flag;           // [16]
-    float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
     float *sL;           // [2][256] -lse of the rows of a phase-2 task (padding: -inf)
+    float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
-    float *xch;          // [2][kEpiWG - 1][128] phase-2 column sums of warpgroups 1..
+    float *xch;          // [kAccBufs][kEpiWG][128] phase-2 partial column sums
+    int *xcnt;           // [kAccBufs][4] arrivals per accumulator and lane quarter
 };
 
 __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
@@ -150,8 +170,10 @@ __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
     return 1024                                   // alignment slack
            + (size_t)2 * nslab * r_pad * 128      // query buffers
            + (size_t)kstages * nslab * kSlabBytes // key ring
-           + kNumBars * 8 + 16 + 64               // barriers, tmem holder, flags
-           + (2 * kEpiWG * 4 * kMaxGroups * 16 + 2 * 256 + 2 * (kEpiWG - 1) * 128 + 4) * 4;
+           + kStageBytes                          // lse merge staging
+           + kCtrlBytes                           // barriers, tmem holder, flags
+           + (2 * 256 + 2 * kEpiWG * 4 * kMaxGroups * 16) * 4 + 16
+           + (kAccBufs * kEpiWG * kTile + kAccBufs * 4) * 4;
 }
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
@@ -165,19 +187,22 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int ks
     off += (uint32_t)(2 * nslab * r_pad * 128);
     s.k = raw + off;
     off += (uint32_t)(kstages * nslab * kSlabBytes);
+    s.stage = reinterpret_cast<float *>(raw + off);
+    off += kStageBytes;
     s.bar = reinterpret_cast<uint64_t *>(raw + off);
-    off += kNumBars * 8;
-    s.tmem = reinterpret_cast<uint32_t *>(raw + off);
-    off += 16;
-    s.flag = reinterpret_cast<int *>(raw + off);
-    off += 64;
+    s.tmem = reinterpret_cast<uint32_t *>(raw + off + kNumBars * 8);
+    s.flag = reinterpret_cast<int *>(raw + off + kNumBars * 8 + 16);
+    static_assert(kNumBars * 8 + 16 + 64 <= kCtrlBytes, "control block");
+    off += kCtrlBytes;
+    s.sL = reinterpret_cast<float *>(raw + off);  // 16-byte aligned: read as float4
+    off += 2 * 256 * 4;
     s.red = reinterpret_cast<float *>(raw + off);
     off += 2 * kEpiWG * 4 * kMaxGroups * 16 * 4;
-    s.sL = reinterpret_cast<float *>(raw + off);
-    off += 2 * 256 * 4;
     s.sLbad = reinterpret_cast<int *>(raw + off);
     off += 16;
     s.xch = reinterpret_cast<float *>(raw + off);
+    off += kAccBufs * kEpiWG * kTile * 4;
+    s.xcnt = reinterpret_cast<int *>(raw + off);
     return s;
 }
 
@@ -343,21 +368,20 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             ptx::mbar_init(&sm.bar[kBarAccEmpty + i], kEpiWarps);
         }
         ptx::mbar_init(&sm.bar[kBarDrain], 1);
+        ptx::mbar_init(&sm.bar[kBarStage], 1);
         for (int i = 0; i < 2; ++i) {
-            ptx::mbar_init(&sm.bar[kBarXFull + i], 4 * (kEpiWG - 1));
-            ptx::mbar_init(&sm.bar[kBarXEmpty + i], 4);
             ptx::mbar_init(&sm.bar[kBarRedFull + i], kEpiWarps);
             ptx::mbar_init(&sm.bar[kBarRedEmpty + i], 1);
             ptx::mbar_init(&sm.bar[kBarLseFull + i], 1);
             ptx::mbar_init(&sm.bar[kBarLseEmpty + i], kEpiWarps);
         }
         flag[kFlagAbort] = 0;
-        flag[kFlagLast] = 0;
-        flag[kFlagWait] = 0;
-        flag[kFlagBad] = 0;
         for (int i = 0; i < kMaxKStages; ++i)
             flag[kFlagKArm + i] = -1;
         flag[kFlagQArm] = flag[kFlagQArm + 1] = -1;
+        flag[kFlagSArm] = -1;
+        for (int i = 0; i < kAccBufs * 4; ++i)
+            sm.xcnt[i] = 0;
         ptx::fence_mbar_init();
     }
     // Query rows R .. r_pad-1 are never written by TMA: zero them once so the padded
@@ -532,98 +556,148 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             drain_bar(&sm.bar[kBarDrain], 0, 2000000000ull);
         }
     } else {
-        // ---- coordinator (warps 2, 3) ----------------------------------------------------
-        // Per step: (a) for the coming phase-2 task, wait until every chunk of its unit has
-        // reported (the unit counter), merge the chunk sums into -lse and hand them to the
-        // epilogue; (b) for the phase-1 task the epilogue is finishing, add its per-warp row
-        // sums, publish them to global memory and count the chunk in.
-        const int ct = threadIdx.x - 64;  // 0 .. kCoordThreads-1
+        // ---- coordinator: warp 2 stages lse, warp 3 hands off row sums ---------------------
+        // Warp 3, per phase-1 task: adds the epilogue warps' row sums of the chunk, publishes
+        // them and counts the chunk into its unit.  Warp 2, per phase-2 task: waits until
+        // every chunk of the task's unit is counted, brings the unit's chunk sums into
+        // shared memory with bulk copies, adds them in chunk order (the same result in every
+        // CTA that needs the unit) and stages -lse for the epilogue.  The two warps never
+        // wait on each other, and a phase-2 task of step t needs only phase-1 tasks of
+        // earlier steps, so the waits cannot form a cycle.
         bool dead = false;
-        auto wait_c = [&](uint64_t *bar, uint32_t parity) {
+        auto wait_w = [&](uint64_t *bar, uint32_t parity) {
             if (!dead) {
                 const bool got = wait_bar(bar, parity, flag, a);
                 dead = !__all_sync(0xffffffffu, got);
             }
             return !dead;
         };
-        int p1c = 0, p2c = 0;
-        for (int t = 0; t <= (int)a.steps; ++t) {
-            Task T;
-            if (get_task(a, t, 1, T)) {
+        if (warp == 2) {
+            // Bounded spin of one lane until every chunk of unit u is counted.
+            auto spin_count = [&](const uint32_t *p) -> bool {
+                const uint64_t t0 = ptx::globaltimer();
+                while (ptx::ld_acquire_u32(p) < (uint32_t)a.nchunks) {
+                    __nanosleep(64);
+                    if (flag[kFlagAbort] || *(volatile uint32_t *)a.status != 0) {
+                        flag[kFlagAbort] = 1;
+                        return false;
+                    }
+                    if (ptx::globaltimer() - t0 > a.timeout_ns) {
+                        flag[kFlagAbort] = 1;
+                        set_status(a.status, DGE_ERR_DEVICE_TIMEOUT);
+                        return false;
+                    }
+                }
+                return true;
+            };
+            const int per_piece = kStageBytes / (a.r4 * 4);  // chunks per bulk copy
+            uint32_t sph = 0;
+            int p2c = 0;
+            for (int t = 0; t <= (int)a.steps; ++t) {
+                Task T;
+                if (!get_task(a, t, 1, T))
+                    continue;
                 const int lb = p2c & 1;
                 const uint32_t lph = (uint32_t)((p2c >> 1) & 1);
                 ++p2c;
-                // Every named barrier below is reached by both warps on every path.
-                const bool ok = wait_c(&sm.bar[kBarLseEmpty + lb], lph ^ 1);
-                if (ct == 0 && ok) {
-                    // Every chunk of the unit has published its row sums.
-                    const uint64_t t0 = ptx::globaltimer();
-                    while (ptx::ld_acquire_u32(&a.count[T.u]) < (uint32_t)a.nchunks) {
-                        __nanosleep(64);
-                        if (flag[kFlagAbort] || *(volatile uint32_t *)a.status != 0) {
-                            flag[kFlagAbort] = 1;
-                            break;
-                        }
-                        if (ptx::globaltimer() - t0 > a.timeout_ns) {
-                            flag[kFlagAbort] = 1;
-                            set_status(a.status, DGE_ERR_DEVICE_TIMEOUT);
-                            break;
-                        }
-                    }
+                if (lane == 0)
+                    trace_at(a, kTrTimeline, 4 * (p2c - 1));
+                int got = wait_w(&sm.bar[kBarLseEmpty + lb], lph ^ 1) ? 1 : 0;
+                if (lane == 0) {
+                    trace_at(a, kTrTimeline, 4 * (p2c - 1) + 1);
+                    got = got && spin_count(&a.count[T.u]);
+                    // The acquire above saw every chunk's sums; the bulk copies below read
+                    // them through the async proxy.
+                    ptx::fence_proxy_async_global();
+                    trace_at(a, kTrTimeline, 4 * (p2c - 1) + 2);
                 }
-                ptx::named_barrier(kBarCoord, kCoordThreads);
-                if (ok) {
-                    float *L = sm.sL + lb * 256;
-                    for (int r = ct; r < a.r_pad; r += kCoordThreads) {
+                got = __shfl_sync(0xffffffffu, got, 0);
+                float Z[kRowsPerLane];
+#pragma unroll
+                for (int i = 0; i < kRowsPerLane; ++i)
+                    Z[i] = 0.f;
+                const float *src = a.part + T.u * a.nchunks * a.r4;
+                for (int c0 = 0; got && c0 < a.nchunks; c0 += per_piece) {
+                    const int nc = min(per_piece, a.nchunks - c0);
+                    __syncwarp();
+                    if (lane == 0) {
+                        // The previous piece's reads (generic proxy) come before the copy.
+                        ptx::fence_proxy_async_smem();
+                        const uint32_t bytes = (uint32_t)(nc * a.r4 * 4);
+                        ptx::mbar_arrive_expect_tx(&sm.bar[kBarStage], bytes);
+                        flag[kFlagSArm] = (int)sph;
+                        ptx::bulk_load(sm.stage, src + (int64_t)c0 * a.r4, bytes, &sm.bar[kBarStage]);
+                    }
+                    if (!wait_w(&sm.bar[kBarStage], sph)) {
+                        got = 0;
+                        break;
+                    }
+                    sph ^= 1;
+                    for (int c = 0; c < nc; ++c)
+#pragma unroll
+                        for (int i = 0; i < kRowsPerLane; ++i) {
+                            const int r = lane + 32 * i;
+                            if (r < g.R)
+                                Z[i] += sm.stage[c * a.r4 + r];
+                        }
+                }
+                bool bad = false;
+                float *L = sm.sL + lb * 256;
+#pragma unroll
+                for (int i = 0; i < kRowsPerLane; ++i) {
+                    const int r = lane + 32 * i;
+                    if (r < a.r_pad) {
                         float v = -INFINITY;
-                        if (r < g.R) {
-                            float Z = 0.f;
-                            for (int c = 0; c < a.nchunks; ++c)
-                                Z += __ldcg(&a.part[(T.u * a.nchunks + c) * g.R + r]);
-                            if (!(Z >= 0x1p-60f && Z < 0x1p126f))
-                                flag[kFlagBad] = 1;
-                            v = -log2f(Z);
+                        if (got && r < g.R) {
+                            if (!(Z[i] >= 0x1p-60f && Z[i] < 0x1p126f))
+                                bad = true;
+                            v = -log2f(Z[i]);
                         }
                         L[r] = v;
                     }
                 }
-                ptx::named_barrier(kBarCoord, kCoordThreads);
-                const int bad = flag[kFlagBad];
-                ptx::named_barrier(kBarCoord, kCoordThreads);
-                if (ct == 0) {
-                    sm.sLbad[lb] = (bad || flag[kFlagAbort] || !ok) ? 1 : 0;
-                    if (bad)
+                bad = __any_sync(0xffffffffu, bad);
+                __syncwarp();
+                if (lane == 0) {
+                    sm.sLbad[lb] = (!got || bad || flag[kFlagAbort]) ? 1 : 0;
+                    if (got && bad)
                         a.ready[T.u] = kReadyBad;  // recomputed after the kernel
-                    flag[kFlagBad] = 0;
+                    trace_at(a, kTrTimeline, 4 * (p2c - 1) + 3);
                     ptx::mbar_arrive(&sm.bar[kBarLseFull + lb]);
                 }
             }
-            if (get_task(a, t, 0, T)) {
+        } else {
+            int p1c = 0;
+            for (int t = 0; t <= (int)a.steps; ++t) {
+                Task T;
+                if (!get_task(a, t, 0, T))
+                    continue;
                 const int rb = p1c & 1;
                 const uint32_t rph = (uint32_t)((p1c >> 1) & 1);
                 ++p1c;
-                const bool ok = wait_c(&sm.bar[kBarRedFull + rb], rph);
+                const bool ok = wait_w(&sm.bar[kBarRedFull + rb], rph);
                 if (ok) {
                     constexpr int W = kMaxGroups * 16;
-                    for (int col = ct; col < g.R; col += kCoordThreads) {
+                    float *dst = a.part + (T.u * a.nchunks + T.chunk) * a.r4;
+                    for (int col = lane; col < g.R; col += 32) {
                         int w = 0;
                         while (w + 1 < kEpiWG && col >= a.gbase[w + 1] * 16)
                             ++w;
                         const int lc = col - a.gbase[w] * 16;
                         const float *rbuf = sm.red + (rb * kEpiWG + w) * 4 * W;
-                        const float sum = rbuf[lc] + rbuf[W + lc] + rbuf[2 * W + lc] + rbuf[3 * W + lc];
-                        a.part[(T.u * a.nchunks + T.chunk) * g.R + col] = sum;
+                        dst[col] = rbuf[lc] + rbuf[W + lc] + rbuf[2 * W + lc] + rbuf[3 * W + lc];
                     }
+                    __threadfence();
                 }
-                ptx::named_barrier(kBarCoord, kCoordThreads);
-                if (ct == 0) {
+                __syncwarp();
+                if (lane == 0) {
                     if (ok) {
-                        // The barrier orders every row-sum store before this cumulative
-                        // release of the chunk count.
+                        // Cumulative release of every lane's sums with the chunk count.
                         ptx::fence_acq_rel_gpu();
                         atomicAdd(&a.count[T.u], 1u);
                     }
                     ptx::mbar_arrive(&sm.bar[kBarRedEmpty + rb]);
+                    trace_step(a, kTrStepTimeline, p1c - 1);
                 }
             }
         }
@@ -631,8 +705,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
     } else {
         ptx::regs_inc<kRegsEpilogue>();
         // ---- epilogue -------------------------------------------------------------------
-        // Every warpgroup reads every tile, its own 16-column groups: phase 1 keeps row sums
-        // in registers, phase 2 forms partial column sums that warpgroup 0 collects.
+        // Every warpgroup reads every tile, its own 16-column groups: phase 1 keeps the row
+        // sums in registers, phase 2 forms partial column sums that the three warps of a
+        // lane quarter combine through shared memory.
         const int ew = warp - kEpiWarp0;         // 0 .. kEpiWarps-1
         const int wg = ew >> 2;                  // warpgroup
         const int quarter = warp & 3;            // TMEM lane quarter of this warp
@@ -640,17 +715,15 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         const int wi = (ew & 3) * 32 + lane;     // thread index within the warpgroup
         const int ng = a.ng[wg];
         const int col_base = a.gbase[wg] * 16;
-        const int ngroups = a.r_pad / 16;
         const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
         const float s2 = g.scale_log2;
         const int first_causal = g.n - g.m;      // keys from here on are not seen by every row
         int tc = 0;   // accumulator tiles consumed (buffer tc % 3, use tc / 3)
-        int xc = 0;   // phase-2 tiles (exchange buffer xc % 2, use xc / 2)
         int p1c = 0;  // phase-1 tasks (row-sum hand-off buffer p1c % 2)
         int p2c = 0;  // phase-2 tasks (-lse buffer p2c % 2)
         bool dead = false;
 
-        long long cy_wa = 0, cy_x = 0, cy_p1e = 0, cy_p2s = 0;
+        long long cy_wa = 0, cy_p1e = 0, cy_p2s = 0;
         const long long cy0 = clock64();
         // Waits for this thread's accumulator and returns false once the CTA is dead
         // (the outcome is warp-uniform: the TMEM loads after it are warp-collective).
@@ -667,12 +740,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         };
         // A bounded, warp-uniform wait on a CTA barrier (false once the CTA is dead).
         auto wait_uniform = [&](uint64_t *bar, uint32_t parity) {
-            const long long c0 = clock64();
             if (!dead) {
                 const bool got = wait_bar(bar, parity, flag, a);
                 dead = !__all_sync(0xffffffffu, got);
             }
-            cy_x += clock64() - c0;
             return !dead;
         };
         auto release_acc = [&](int ab, uint32_t count) {
@@ -711,7 +782,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                                 if (gi < ng) {
                                     float v[16];
                                     ptx::tmem_ld16(tbase + gi * 16, v);
-                                    ptx::tmem_ld_wait();
+                                    ptx::tmem_ld_wait_dep(v);
                                     rows_add(z[gi], v, s2, valid, causal, key, first_causal,
                                              col_base + gi * 16, g.m);
                                 }
@@ -752,18 +823,30 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 } else {
                     const long long c_start = clock64();
                     // ---------------- phase 2: column sums of this chunk ----------------
-                    // The coordinator warps have put -lse of this unit's rows in sL[lb].
+                    // The coordinator warp has put -lse of this unit's rows in sL[lb]; this
+                    // warpgroup's columns go to registers and the buffer is released.
                     const int lb = p2c & 1;
                     const uint32_t lph = (uint32_t)((p2c >> 1) & 1);
+                    ++p2c;
+                    if (ew == 0 && lane == 0)
+                        trace_at(a, kTrTimeline, 2048 + 2 * (p2c - 1));
                     float nL[kMaxGroups][16];
                     bool task_ok = false;
                     if (wait_uniform(&sm.bar[kBarLseFull + lb], lph)) {
-                        const float *L = sm.sL + lb * 256 + col_base;
+                        const float4 *L4 =
+                            reinterpret_cast<const float4 *>(sm.sL + lb * 256 + col_base);
 #pragma unroll
                         for (int gi = 0; gi < kMaxGroups; ++gi)
 #pragma unroll
-                            for (int c = 0; c < 16; ++c)
-                                nL[gi][c] = gi < ng ? L[gi * 16 + c] : -INFINITY;
+                            for (int i = 0; i < 4; ++i) {
+                                const float4 q = gi < ng ? L4[gi * 4 + i]
+                                                         : make_float4(-INFINITY, -INFINITY,
+                                                                       -INFINITY, -INFINITY);
+                                nL[gi][4 * i] = q.x;
+                                nL[gi][4 * i + 1] = q.y;
+                                nL[gi][4 * i + 2] = q.z;
+                                nL[gi][4 * i + 3] = q.w;
+                            }
                         task_ok = sm.sLbad[lb] == 0;
                         __syncwarp();
                         if (lane == 0)
@@ -775,10 +858,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                             for (int c = 0; c < 16; ++c)
                                 nL[gi][c] = -INFINITY;
                     }
+                    if (ew == 0 && lane == 0)
+                        trace_at(a, kTrTimeline, 2048 + 2 * (p2c - 1) + 1);
                     task_ok = task_ok && !dead;
-                    ++p2c;
                     cy_p2s += clock64() - c_start;
-                    for (int tile = 0; tile < T.ntiles; ++tile, ++tc, ++xc) {
+                    for (int tile = 0; tile < T.ntiles; ++tile, ++tc) {
                         const int ab = tc % kAccBufs;
                         const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
                         const int tile0 = T.k_lo + tile * kTile;
@@ -793,43 +877,40 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                                 if (gi < ng) {
                                     float v[16];
                                     ptx::tmem_ld16(tbase + gi * 16, v);
-                                    ptx::tmem_ld_wait();
+                                    ptx::tmem_ld_wait_dep(v);
                                     col_add(acc, v, nL[gi], s2, causal, key, first_causal,
                                             col_base + gi * 16, g.m);
                                 }
                         }
-                        release_acc(ab, 1u);
-                        // Warpgroups 1.. hand their partial sums to warpgroup 0 through a
-                        // double-buffered exchange; warpgroup 0 adds them in a fixed order.
-                        const int xb = xc & 1;
-                        const uint32_t xph = (uint32_t)((xc >> 1) & 1);
-                        float *xrow = sm.xch + xb * (kEpiWG - 1) * kTile;
-                        if (wg > 0) {
-                            if (wait_uniform(&sm.bar[kBarXEmpty + xb], xph ^ 1)) {
-                                xrow[(wg - 1) * kTile + kl] = acc.x + acc.y;
-                                __syncwarp();
-                                if (lane == 0)
-                                    ptx::mbar_arrive(&sm.bar[kBarXFull + xb]);
-                            }
-                        } else {
-                            if (wait_uniform(&sm.bar[kBarXFull + xb], xph)) {
-                                float total = acc.x + acc.y;
-#pragma unroll
-                                for (int w = 0; w < kEpiWG - 1; ++w)
-                                    total += xrow[w * kTile + kl];
-                                if (task_ok && key < T.k_hi)
-                                    a.raw[T.u * g.P + key] = total;
-                                __syncwarp();
-                                if (lane == 0)
-                                    ptx::mbar_arrive(&sm.bar[kBarXEmpty + xb]);
-                            }
+                        // The three warps of this lane quarter (one per warpgroup) leave their
+                        // partial sums in shared memory; whichever comes last adds them in
+                        // warpgroup order and stores the key's score.  Nobody waits: a slot is
+                        // rewritten only after accumulator ab is refilled, which needs every
+                        // warp's release below, the last warp's after its reads.
+                        float *xs = sm.xch + ab * kEpiWG * kTile;
+                        xs[wg * kTile + kl] = acc.x + acc.y;
+                        __syncwarp();
+                        int last = 0;
+                        if (lane == 0) {
+                            __threadfence_block();
+                            last = atomicAdd(&sm.xcnt[ab * 4 + quarter], 1) % kEpiWG == kEpiWG - 1;
+                            __threadfence_block();
                         }
+                        last = __shfl_sync(0xffffffffu, last, 0);
+                        if (last) {
+                            float total = xs[kl];
+#pragma unroll
+                            for (int w = 1; w < kEpiWG; ++w)
+                                total += xs[w * kTile + kl];
+                            if (task_ok && key < T.k_hi)
+                                a.raw[T.u * g.P + key] = total;
+                        }
+                        release_acc(ab, 1u);
                     }
                 }
             }
         if (ew == 0 && lane == 0) {
             trace_put(a, kTrEpiWaitAcc, cy_wa);
-            trace_put(a, kTrEpiExchange, cy_x);
             trace_put(a, kTrEpiP1End, cy_p1e);
             trace_put(a, kTrEpiP2Start, cy_p2s);
             trace_put(a, kTrEpiTotal, clock64() - cy0);
@@ -846,6 +927,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         for (int i = 0; i < 2; ++i)
             if (flag[kFlagQArm + i] >= 0)
                 drain_bar(&sm.bar[kBarQFull + i], (uint32_t)flag[kFlagQArm + i], 1000000000ull);
+        if (flag[kFlagSArm] >= 0)
+            drain_bar(&sm.bar[kBarStage], (uint32_t)flag[kFlagSArm], 1000000000ull);
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -910,7 +993,8 @@ void tc_set_trace(unsigned long long *buffer, int cta)
 bool tc_supported(const Geometry &g)
 {
     if (g.variant != DGE_VARIANT_SCORED || (g.d != 64 && g.d != 128) ||
-        g.R > kEpiWG * kMaxGroups * 16 || g.m > 256 || g.G > 256)
+        g.R > kEpiWG * kMaxGroups * 16 || g.R > 32 * kRowsPerLane ||
+        (size_t)((g.R + 3) & ~3) * 4 > (size_t)kStageBytes || g.m > 256 || g.G > 256)
         return false;
     int dev = 0, major = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -923,6 +1007,7 @@ TcPlan tc_plan(const Geometry &g)
 {
     TcPlan p;
     p.r_pad = (g.R + 15) & ~15;
+    p.r4 = (g.R + 3) & ~3;
     p.nslab = g.d / 64;
     p.chunk_keys = 1024;
     p.nchunks = (g.n + p.chunk_keys - 1) / p.chunk_keys;
@@ -956,6 +1041,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     TcArgs a;
     a.g = g;
     a.r_pad = plan.r_pad;
+    a.r4 = plan.r4;
     a.acc_stride = (plan.r_pad + 31) & ~31;
     a.nslab = plan.nslab;
     a.kstages = plan.kstages;
@@ -969,7 +1055,9 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
         base += a.ng[w];
     }
     const int64_t grid = a.items < sms ? a.items : sms;
-    a.steps = (a.items + grid - 1) / grid;
+    a.lag = plan.nchunks - 1;
+    // Phase 2 of the last item runs in step `steps`: (steps - 1) * grid + s - lag covers it.
+    a.steps = (a.items + a.lag + grid - 1) / grid;
     a.part = buf.part;
     a.lse2 = buf.lse2;
     a.raw = buf.raw;
