@@ -235,10 +235,13 @@ int dge_profile_end(dge_kernel_time *out, int capacity, int *count);
  * phase-1 task i into the unit.  Slot 13, for CTA `cta` only: entry 4i .. 4i+3 when
  * its coordinator starts staging phase-2 task i, has the buffer, sees every chunk
  * of the unit counted and has staged lse; entry 2048 + 2i / 2i+1 when its first
- * epilogue warp starts / ends waiting for that lse.  `bytes` must cover the slots;
+ * epilogue warp starts / ends waiting for that lse.  Slots 17 .. 19: the first
+ * epilogue warp's cycles reading accumulators and adding exponentials, in the
+ * phase-2 exchange and in releasing accumulators; 16 and 20 .. 23 unused.  `bytes`
+ * must cover the slots;
  * pass NULL to stop.  Host-side state, per process.
  */
-#define DGE_TRACE_SLOTS 16
+#define DGE_TRACE_SLOTS 24
 #define DGE_TRACE_LEN 4096
 int dge_trace_set(void *buffer, size_t bytes, int cta);
 

@@ -178,7 +178,7 @@ def dge_profile_end(capacity: int = 32) -> list:
             for i in range(min(count.value, capacity))]
 
 
-TRACE_SLOTS, TRACE_LEN = 16, 4096
+TRACE_SLOTS, TRACE_LEN = 24, 4096
 
 
 def dge_trace_set(buffer: int, nbytes: int, cta: int = 0) -> None:

@@ -59,9 +59,9 @@ constexpr uint32_t kReadyBad = 2;          // unit left fp32's range: recomputed
 // Barrier slots.
 constexpr int kBarKFull = 0, kBarKEmpty = 4, kBarQFull = 8, kBarQEmpty = 10, kBarAccFull = 12,
               kBarAccEmpty = 15, kBarDrain = 18, kBarRedFull = 19, kBarRedEmpty = 21,
-              kBarLseFull = 23, kBarLseEmpty = 25, kBarStage = 27, kNumBars = 28;
+              kBarLseFull = 23, kBarLseEmpty = 25, kBarStage = 27, kBarXch = 28, kNumBars = 40;
 constexpr int kStageBytes = 12288;        // chunk sums of a unit, staged for the lse merge
-constexpr int kCtrlBytes = 320;            // barriers, TMEM address, flags (16-byte multiple)
+constexpr int kCtrlBytes = 400;            // barriers, TMEM address, flags (16-byte multiple)
 constexpr int kRowsPerLane = 5;           // rows of the lse merge per lane (R <= 160)
 // Flag slots (ints): abort, then the parity of the last arm of every key stage, query
 // buffer and the staging buffer (-1 = never armed) for the drain.
@@ -93,28 +93,41 @@ struct TcArgs {
 enum TraceSlot {
     kTrMmaWaitQ = 0, kTrMmaWaitK, kTrMmaWaitAcc, kTrMmaIssue, kTrMmaCommit, kTrMmaTotal,
     kTrProdWaitQ, kTrProdWaitK, kTrProdTotal, kTrEpiWaitAcc, kTrStepTimeline, kTrEpiP1End,
-    kTrEpiP2Start, kTrTimeline, kTrEpiTotal, kTrTiles
+    kTrEpiP2Start, kTrTimeline, kTrEpiTotal, kTrTiles, kTrUnused16, kTrEpiMath, kTrEpiXch,
+    kTrEpiRelease
 };
 
+template <bool kTr>
 __device__ __forceinline__ void trace_put(const TcArgs &a, int slot, long long v)
 {
-    if (a.trace && blockIdx.x < DGE_TRACE_LEN)
+    if (kTr && a.trace && blockIdx.x < DGE_TRACE_LEN)
         a.trace[slot * DGE_TRACE_LEN + blockIdx.x] = (unsigned long long)v;
 }
 
 // Timeline of CTA a.trace_cta: global-timer stamps (ns) at index i of a timeline slot.
+template <bool kTr>
 __device__ __forceinline__ void trace_at(const TcArgs &a, int slot, int i)
 {
-    if (a.trace && (int)blockIdx.x == a.trace_cta && i >= 0 && i < DGE_TRACE_LEN)
+    if (kTr && a.trace && (int)blockIdx.x == a.trace_cta && i >= 0 && i < DGE_TRACE_LEN)
         a.trace[slot * DGE_TRACE_LEN + i] = ptx::globaltimer();
 }
 
 // Step timeline of every CTA: global-timer stamp of its phase-1 task i at i * grid + cta.
+template <bool kTr>
 __device__ __forceinline__ void trace_step(const TcArgs &a, int slot, int i)
 {
     const int64_t idx = (int64_t)i * gridDim.x + blockIdx.x;
-    if (a.trace && idx < DGE_TRACE_LEN)
+    if (kTr && a.trace && idx < DGE_TRACE_LEN)
         a.trace[slot * DGE_TRACE_LEN + idx] = ptx::globaltimer();
+}
+
+// SM clock for the cycle accounting; a constant 0 in the kernel built without it.
+template <bool kTr>
+__device__ __forceinline__ long long tclock()
+{
+    if (kTr)
+        return clock64();
+    return 0;
 }
 
 struct Task {
@@ -162,7 +175,6 @@ struct Smem {
     float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
     float *xch;          // [kAccBufs][kEpiWG][128] phase-2 partial column sums
-    int *xcnt;           // [kAccBufs][4] arrivals per accumulator and lane quarter
 };
 
 __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
@@ -173,7 +185,7 @@ __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
            + kStageBytes                          // lse merge staging
            + kCtrlBytes                           // barriers, tmem holder, flags
            + (2 * 256 + 2 * kEpiWG * 4 * kMaxGroups * 16) * 4 + 16
-           + (kAccBufs * kEpiWG * kTile + kAccBufs * 4) * 4;
+           + kAccBufs * kEpiWG * kTile * 4;
 }
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
@@ -201,8 +213,6 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int ks
     s.sLbad = reinterpret_cast<int *>(raw + off);
     off += 16;
     s.xch = reinterpret_cast<float *>(raw + off);
-    off += kAccBufs * kEpiWG * kTile * 4;
-    s.xcnt = reinterpret_cast<int *>(raw + off);
     return s;
 }
 
@@ -342,6 +352,25 @@ __device__ __forceinline__ void col_add(float2 &acc, const float (&v)[16], const
     }
 }
 
+// Runs f(gi, v) over this warp's lane quarter of 16-column groups gi = 0 .. ng-1 (ng <=
+// kMaxGroups, warp-uniform) read from TMEM, one group per round trip.  (Keeping the next
+// group's load in flight while f runs measured markedly slower.)
+template <typename F>
+__device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
+{
+#pragma unroll
+    for (int gi = 0; gi < kMaxGroups; ++gi)
+        if (gi < ng) {
+            float v[16];
+            ptx::tmem_ld16(tbase + gi * 16, v);
+            ptx::tmem_ld_wait_dep(v);
+            f(gi, v);
+        }
+}
+
+// kTr: with the cycle accounting and timelines of dge_trace_set (a separate build, so the
+// clock reads cost nothing when tracing is off).
+template <bool kTr>
 __global__ void __launch_bounds__(kThreads, 1)
 score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
                 const TcArgs a)
@@ -380,8 +409,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             flag[kFlagKArm + i] = -1;
         flag[kFlagQArm] = flag[kFlagQArm + 1] = -1;
         flag[kFlagSArm] = -1;
+        // Phase-2 exchange: one barrier per accumulator and lane quarter, one arrival per
+        // warpgroup.
         for (int i = 0; i < kAccBufs * 4; ++i)
-            sm.xcnt[i] = 0;
+            ptx::mbar_init(&sm.bar[kBarXch + i], kEpiWG);
         ptx::fence_mbar_init();
     }
     // Query rows R .. r_pad-1 are never written by TMA: zero them once so the padded
@@ -421,7 +452,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             int ks = 0, qb = 0;
             uint32_t kph = 0, qph = 0;
             long long cy_wq = 0, cy_wk = 0;
-            const long long cy0 = clock64();
+            const long long cy0 = tclock<kTr>();
             bool ok = true;
             for (int64_t t = 0; ok && t <= a.steps; ++t)
                 for (int j = 0; ok && j < 2; ++j) {
@@ -430,12 +461,12 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         continue;
                     int l, bb, h;
                     unit_coords(g, T.u, l, bb, h);
-                    long long c0 = clock64();
+                    long long c0 = tclock<kTr>();
                     if (!wait_bar(&sm.bar[kBarQEmpty + qb], qph ^ 1, flag, a)) {
                         ok = false;
                         break;
                     }
-                    cy_wq += clock64() - c0;
+                    cy_wq += tclock<kTr>() - c0;
                     ptx::mbar_arrive_expect_tx(&sm.bar[kBarQFull + qb],
                                                (uint32_t)a.nslab * 128u * (uint32_t)g.R);
                     flag[kFlagQArm + qb] = (int)qph;
@@ -448,12 +479,12 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         qph ^= 1;
                     const uint64_t pol = T.phase == 2 ? drop : keep;
                     for (int tile = 0; tile < T.ntiles; ++tile) {
-                        c0 = clock64();
+                        c0 = tclock<kTr>();
                         if (!wait_bar(&sm.bar[kBarKEmpty + ks], kph ^ 1, flag, a)) {
                             ok = false;
                             break;
                         }
-                        cy_wk += clock64() - c0;
+                        cy_wk += tclock<kTr>() - c0;
                         ptx::mbar_arrive_expect_tx(&sm.bar[kBarKFull + ks],
                                                    (uint32_t)a.nslab * kSlabBytes);
                         flag[kFlagKArm + ks] = (int)kph;
@@ -467,9 +498,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         }
                     }
                 }
-            trace_put(a, kTrProdWaitQ, cy_wq);
-            trace_put(a, kTrProdWaitK, cy_wk);
-            trace_put(a, kTrProdTotal, clock64() - cy0);
+            trace_put<kTr>(a, kTrProdWaitQ, cy_wq);
+            trace_put<kTr>(a, kTrProdWaitK, cy_wk);
+            trace_put<kTr>(a, kTrProdTotal, tclock<kTr>() - cy0);
         }
     } else if (warp == 1) {
         // ---- MMA issuer -----------------------------------------------------------------
@@ -479,35 +510,35 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             uint32_t kph = 0, qph = 0;
             int64_t tc = 0;  // accumulator sequence number: buffer tc % 3, use tc / 3
             long long cy_wq = 0, cy_wk = 0, cy_wa = 0, cy_is = 0, cy_cm = 0;
-            const long long cy0 = clock64();
+            const long long cy0 = tclock<kTr>();
             bool ok = true;
             for (int64_t t = 0; ok && t <= a.steps; ++t)
                 for (int j = 0; ok && j < 2; ++j) {
                     Task T;
                     if (!get_task(a, t, j, T))
                         continue;
-                    long long c0 = clock64();
+                    long long c0 = tclock<kTr>();
                     if (!wait_bar(&sm.bar[kBarQFull + qb], qph, flag, a)) {
                         ok = false;
                         break;
                     }
-                    cy_wq += clock64() - c0;
+                    cy_wq += tclock<kTr>() - c0;
                     const uint32_t qbase = ptx::smem_addr(sm.q + (size_t)qb * a.nslab * q_slab_bytes);
                     for (int tile = 0; tile < T.ntiles; ++tile, ++tc) {
                         const int ab = (int)(tc % kAccBufs);
                         const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
-                        c0 = clock64();
+                        c0 = tclock<kTr>();
                         if (!wait_bar(&sm.bar[kBarKFull + ks], kph, flag, a)) {
                             ok = false;
                             break;
                         }
-                        long long c1 = clock64();
+                        long long c1 = tclock<kTr>();
                         cy_wk += c1 - c0;
                         if (!wait_bar(&sm.bar[kBarAccEmpty + ab], aph ^ 1, flag, a)) {
                             ok = false;
                             break;
                         }
-                        c0 = clock64();
+                        c0 = tclock<kTr>();
                         cy_wa += c0 - c1;
                         ptx::tc_fence_after();
                         // Descriptors are linear in the start address (bits 0..13 hold
@@ -527,11 +558,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                                               kk > 0 ? 1u : 0u);
                             }
                         }
-                        c1 = clock64();
+                        c1 = tclock<kTr>();
                         cy_is += c1 - c0;
                         ptx::mma_commit(&sm.bar[kBarKEmpty + ks]);
                         ptx::mma_commit(&sm.bar[kBarAccFull + ab]);
-                        cy_cm += clock64() - c1;
+                        cy_cm += tclock<kTr>() - c1;
                         if (++ks == a.kstages) {
                             ks = 0;
                             kph ^= 1;
@@ -544,13 +575,13 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     if (qb == 0)
                         qph ^= 1;
                 }
-            trace_put(a, kTrMmaWaitQ, cy_wq);
-            trace_put(a, kTrMmaWaitK, cy_wk);
-            trace_put(a, kTrMmaWaitAcc, cy_wa);
-            trace_put(a, kTrMmaIssue, cy_is);
-            trace_put(a, kTrMmaCommit, cy_cm);
-            trace_put(a, kTrMmaTotal, clock64() - cy0);
-            trace_put(a, kTrTiles, tc);
+            trace_put<kTr>(a, kTrMmaWaitQ, cy_wq);
+            trace_put<kTr>(a, kTrMmaWaitK, cy_wk);
+            trace_put<kTr>(a, kTrMmaWaitAcc, cy_wa);
+            trace_put<kTr>(a, kTrMmaIssue, cy_is);
+            trace_put<kTr>(a, kTrMmaCommit, cy_cm);
+            trace_put<kTr>(a, kTrMmaTotal, tclock<kTr>() - cy0);
+            trace_put<kTr>(a, kTrTiles, tc);
             // Every MMA issued so far completes before the drain barrier fires.
             ptx::mma_commit(&sm.bar[kBarDrain]);
             drain_bar(&sm.bar[kBarDrain], 0, 2000000000ull);
@@ -601,15 +632,15 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 const uint32_t lph = (uint32_t)((p2c >> 1) & 1);
                 ++p2c;
                 if (lane == 0)
-                    trace_at(a, kTrTimeline, 4 * (p2c - 1));
+                    trace_at<kTr>(a, kTrTimeline, 4 * (p2c - 1));
                 int got = wait_w(&sm.bar[kBarLseEmpty + lb], lph ^ 1) ? 1 : 0;
                 if (lane == 0) {
-                    trace_at(a, kTrTimeline, 4 * (p2c - 1) + 1);
+                    trace_at<kTr>(a, kTrTimeline, 4 * (p2c - 1) + 1);
                     got = got && spin_count(&a.count[T.u]);
                     // The acquire above saw every chunk's sums; the bulk copies below read
                     // them through the async proxy.
                     ptx::fence_proxy_async_global();
-                    trace_at(a, kTrTimeline, 4 * (p2c - 1) + 2);
+                    trace_at<kTr>(a, kTrTimeline, 4 * (p2c - 1) + 2);
                 }
                 got = __shfl_sync(0xffffffffu, got, 0);
                 float Z[kRowsPerLane];
@@ -662,7 +693,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     sm.sLbad[lb] = (!got || bad || flag[kFlagAbort]) ? 1 : 0;
                     if (got && bad)
                         a.ready[T.u] = kReadyBad;  // recomputed after the kernel
-                    trace_at(a, kTrTimeline, 4 * (p2c - 1) + 3);
+                    trace_at<kTr>(a, kTrTimeline, 4 * (p2c - 1) + 3);
                     ptx::mbar_arrive(&sm.bar[kBarLseFull + lb]);
                 }
             }
@@ -697,7 +728,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         atomicAdd(&a.count[T.u], 1u);
                     }
                     ptx::mbar_arrive(&sm.bar[kBarRedEmpty + rb]);
-                    trace_step(a, kTrStepTimeline, p1c - 1);
+                    trace_step<kTr>(a, kTrStepTimeline, p1c - 1);
                 }
             }
         }
@@ -712,7 +743,6 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         const int wg = ew >> 2;                  // warpgroup
         const int quarter = warp & 3;            // TMEM lane quarter of this warp
         const int kl = quarter * 32 + lane;      // key within the tile
-        const int wi = (ew & 3) * 32 + lane;     // thread index within the warpgroup
         const int ng = a.ng[wg];
         const int col_base = a.gbase[wg] * 16;
         const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
@@ -723,19 +753,19 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         int p2c = 0;  // phase-2 tasks (-lse buffer p2c % 2)
         bool dead = false;
 
-        long long cy_wa = 0, cy_p1e = 0, cy_p2s = 0;
-        const long long cy0 = clock64();
+        long long cy_wa = 0, cy_p1e = 0, cy_p2s = 0, cy_math = 0, cy_xch = 0, cy_rel = 0;
+        const long long cy0 = tclock<kTr>();
         // Waits for this thread's accumulator and returns false once the CTA is dead
         // (the outcome is warp-uniform: the TMEM loads after it are warp-collective).
         auto acquire_acc = [&](int ab, uint32_t aph) {
-            const long long c0 = clock64();
+            const long long c0 = tclock<kTr>();
             if (!dead) {
                 const bool got = wait_bar(&sm.bar[kBarAccFull + ab], aph, flag, a);
                 dead = !__all_sync(0xffffffffu, got);
             }
             if (!dead)
                 ptx::tc_fence_after();
-            cy_wa += clock64() - c0;
+            cy_wa += tclock<kTr>() - c0;
             return !dead;
         };
         // A bounded, warp-uniform wait on a CTA barrier (false once the CTA is dead).
@@ -747,10 +777,12 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             return !dead;
         };
         auto release_acc = [&](int ab, uint32_t count) {
+            const long long c0 = tclock<kTr>();
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0 && !dead)
                 ptx::mbar_arrive_cnt(&sm.bar[kBarAccEmpty + ab], count);
+            cy_rel += tclock<kTr>() - c0;
         };
 
         for (int t = 0; t <= (int)a.steps; ++t)
@@ -774,22 +806,22 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         const bool valid = key < T.k_hi;
                         const bool causal = tile0 + kTile > first_causal;
                         if (acquire_acc(ab, aph)) {
-                            // One 16-column group per TMEM round trip (a few tens of cycles).
+                            // All of this warp's columns in one TMEM round trip.
                             const uint32_t tbase =
                                 tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
+                            const long long c0 = tclock<kTr>();
+                            for_groups(tbase, ng, [&](int gi, const float(&v)[16]) {
 #pragma unroll
-                            for (int gi = 0; gi < kMaxGroups; ++gi)
-                                if (gi < ng) {
-                                    float v[16];
-                                    ptx::tmem_ld16(tbase + gi * 16, v);
-                                    ptx::tmem_ld_wait_dep(v);
-                                    rows_add(z[gi], v, s2, valid, causal, key, first_causal,
-                                             col_base + gi * 16, g.m);
-                                }
+                                for (int gj = 0; gj < kMaxGroups; ++gj)
+                                    if (gj == gi)
+                                        rows_add(z[gj], v, s2, valid, causal, key, first_causal,
+                                                 col_base + gj * 16, g.m);
+                            });
+                            cy_math += tclock<kTr>() - c0;
                         }
                         release_acc(ab, 1u);
                     }
-                    const long long c_end = clock64();
+                    const long long c_end = tclock<kTr>();
                     // Sums over this warp's 32 keys, handed to the coordinator warps through
                     // a double-buffered area (they add the warps in a fixed order).
                     const int rb = p1c & 1;
@@ -819,9 +851,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                             ptx::mbar_arrive(&sm.bar[kBarRedFull + rb]);
                     }
                     ++p1c;
-                    cy_p1e += clock64() - c_end;
+                    cy_p1e += tclock<kTr>() - c_end;
                 } else {
-                    const long long c_start = clock64();
+                    const long long c_start = tclock<kTr>();
                     // ---------------- phase 2: column sums of this chunk ----------------
                     // The coordinator warp has put -lse of this unit's rows in sL[lb]; this
                     // warpgroup's columns go to registers and the buffer is released.
@@ -829,7 +861,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     const uint32_t lph = (uint32_t)((p2c >> 1) & 1);
                     ++p2c;
                     if (ew == 0 && lane == 0)
-                        trace_at(a, kTrTimeline, 2048 + 2 * (p2c - 1));
+                        trace_at<kTr>(a, kTrTimeline, 2048 + 2 * (p2c - 1));
                     float nL[kMaxGroups][16];
                     bool task_ok = false;
                     if (wait_uniform(&sm.bar[kBarLseFull + lb], lph)) {
@@ -859,9 +891,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                                 nL[gi][c] = -INFINITY;
                     }
                     if (ew == 0 && lane == 0)
-                        trace_at(a, kTrTimeline, 2048 + 2 * (p2c - 1) + 1);
+                        trace_at<kTr>(a, kTrTimeline, 2048 + 2 * (p2c - 1) + 1);
                     task_ok = task_ok && !dead;
-                    cy_p2s += clock64() - c_start;
+                    cy_p2s += tclock<kTr>() - c_start;
                     for (int tile = 0; tile < T.ntiles; ++tile, ++tc) {
                         const int ab = tc % kAccBufs;
                         const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
@@ -872,31 +904,35 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         if (acquire_acc(ab, aph)) {
                             const uint32_t tbase =
                                 tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
+                            const long long c0 = tclock<kTr>();
+                            for_groups(tbase, ng, [&](int gi, const float(&v)[16]) {
 #pragma unroll
-                            for (int gi = 0; gi < kMaxGroups; ++gi)
-                                if (gi < ng) {
-                                    float v[16];
-                                    ptx::tmem_ld16(tbase + gi * 16, v);
-                                    ptx::tmem_ld_wait_dep(v);
-                                    col_add(acc, v, nL[gi], s2, causal, key, first_causal,
-                                            col_base + gi * 16, g.m);
-                                }
+                                for (int gj = 0; gj < kMaxGroups; ++gj)
+                                    if (gj == gi)
+                                        col_add(acc, v, nL[gj], s2, causal, key, first_causal,
+                                                col_base + gj * 16, g.m);
+                            });
+                            cy_math += tclock<kTr>() - c0;
                         }
                         // The three warps of this lane quarter (one per warpgroup) leave their
                         // partial sums in shared memory; whichever comes last adds them in
                         // warpgroup order and stores the key's score.  Nobody waits: a slot is
                         // rewritten only after accumulator ab is refilled, which needs every
                         // warp's release below, the last warp's after its reads.
+                        const long long cx = tclock<kTr>();
                         float *xs = sm.xch + ab * kEpiWG * kTile;
                         xs[wg * kTile + kl] = acc.x + acc.y;
                         __syncwarp();
+                        // The arrival releases this warp's sums; a warp that finds the phase
+                        // complete right after its own arrival has all three (two warps may
+                        // both find it so: they store the same value).
                         int last = 0;
                         if (lane == 0) {
-                            __threadfence_block();
-                            last = atomicAdd(&sm.xcnt[ab * 4 + quarter], 1) % kEpiWG == kEpiWG - 1;
-                            __threadfence_block();
+                            uint64_t *xb = &sm.bar[kBarXch + ab * 4 + quarter];
+                            last = ptx::mbar_test_token(xb, ptx::mbar_arrive_token(xb)) ? 1 : 0;
                         }
                         last = __shfl_sync(0xffffffffu, last, 0);
+                        __syncwarp();  // lane 0's acquire orders the other lanes' reads
                         if (last) {
                             float total = xs[kl];
 #pragma unroll
@@ -905,15 +941,19 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                             if (task_ok && key < T.k_hi)
                                 a.raw[T.u * g.P + key] = total;
                         }
+                        cy_xch += tclock<kTr>() - cx;
                         release_acc(ab, 1u);
                     }
                 }
             }
         if (ew == 0 && lane == 0) {
-            trace_put(a, kTrEpiWaitAcc, cy_wa);
-            trace_put(a, kTrEpiP1End, cy_p1e);
-            trace_put(a, kTrEpiP2Start, cy_p2s);
-            trace_put(a, kTrEpiTotal, clock64() - cy0);
+            trace_put<kTr>(a, kTrEpiWaitAcc, cy_wa);
+            trace_put<kTr>(a, kTrEpiP1End, cy_p1e);
+            trace_put<kTr>(a, kTrEpiP2Start, cy_p2s);
+            trace_put<kTr>(a, kTrEpiMath, cy_math);
+            trace_put<kTr>(a, kTrEpiXch, cy_xch);
+            trace_put<kTr>(a, kTrEpiRelease, cy_rel);
+            trace_put<kTr>(a, kTrEpiTotal, tclock<kTr>() - cy0);
         }
     }
 
@@ -1068,7 +1108,8 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.trace = g_trace;
     a.trace_cta = g_trace_cta;
 
-    void (*kernel)(const CUtensorMap, const CUtensorMap, const TcArgs) = score_tc_kernel;
+    void (*kernel)(const CUtensorMap, const CUtensorMap, const TcArgs) =
+        a.trace ? score_tc_kernel<true> : score_tc_kernel<false>;
     err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                (int)plan.smem);
     if (err != cudaSuccess)

@@ -48,6 +48,28 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
                  : "memory");
 }
 
+// Arrive (release, CTA scope) and return the barrier state token of this arrival.
+__device__ __forceinline__ uint64_t mbar_arrive_token(uint64_t *bar)
+{
+    uint64_t st;
+    asm volatile("mbarrier.arrive.shared::cta.b64 %0, [%1];" : "=l"(st) : "r"(smem_addr(bar)) : "memory");
+    return st;
+}
+
+// Non-blocking (acquire, CTA scope): has the phase of the token's arrival completed?
+__device__ __forceinline__ bool mbar_test_token(uint64_t *bar, uint64_t state)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.b32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "l"(state)
+        : "memory");
+    return ok != 0;
+}
+
 // Test for completion of the phase with parity `parity`; the thread may be suspended in
 // hardware (up to a time hint of about a millisecond) until the phase completes, so waiting
 // warps do not spin on the issue slots.
@@ -201,6 +223,15 @@ __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.
 
 // Waits for this thread's TMEM loads and marks the 16 registers of one of them as written
 // by the wait, so no use of them can be scheduled before it.
+// Marks 16 registers as written here (after a tmem_ld_wait_dep of a load issued with them).
+__device__ __forceinline__ void reg_dep(float (&v)[16])
+{
+    asm volatile(""
+                 : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]),
+                   "+f"(v[6]), "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]),
+                   "+f"(v[12]), "+f"(v[13]), "+f"(v[14]), "+f"(v[15]));
+}
+
 __device__ __forceinline__ void tmem_ld_wait_dep(float (&v)[16])
 {
     asm volatile("tcgen05.wait::ld.sync.aligned;"
