@@ -228,16 +228,18 @@ int dge_profile_end(dge_kernel_time *out, int capacity, int *count);
  * waiting for key tiles, 2 MMA waiting for a free accumulator, 3 MMA issuing, 4 MMA
  * committing, 5 MMA total, 6 producer waiting for a query buffer, 7 producer waiting
  * for a key stage, 8 producer total, 9 first epilogue warp waiting for accumulators,
- * 10 step timeline (below), 11 its phase-1 task ends (row-sum hand-off), 12 its
- * phase-2 task starts (waiting for the staged lse), 13 timeline (below), 14 its
- * total, 15 tiles issued.  Timelines hold global-timer stamps (ns).  Slot 10 entry
- * i * grid + c (while below DGE_TRACE_LEN): when CTA c counted the chunk of its
- * phase-1 task i into the unit.  Slot 13, for CTA `cta` only: entry 4i .. 4i+3 when
+ * 10 its phase-2 cycles reading accumulators and adding exponentials, 11 its
+ * phase-1 task ends (row-sum hand-off), 12 its phase-2 task starts (waiting for the
+ * staged lse), 13 timeline (below), 14 its total, 15 tiles issued.  Timelines hold
+ * global-timer stamps (ns).  Slot 13, for CTA `cta` only: entry 4i .. 4i+3 when
  * its coordinator starts staging phase-2 task i, has the buffer, sees every chunk
  * of the unit counted and has staged lse; entry 2048 + 2i / 2i+1 when its first
  * epilogue warp starts / ends waiting for that lse.  Slots 17 .. 19: the first
- * epilogue warp's cycles reading accumulators and adding exponentials, in the
- * phase-2 exchange and in releasing accumulators; 16 and 20 .. 23 unused.  `bytes`
+ * epilogue warp's phase-1 cycles reading accumulators and adding exponentials, its
+ * cycles in the phase-2 exchange and in releasing accumulators.  Per-tile timelines of CTA `cta`,
+ * entry i for its i-th key tile: slot 16 when the producer issues its copy, 20 when
+ * the MMA warp sees it landed, 21 when its accumulator is free, 22 when its MMAs
+ * are issued and committed, 23 when the first epilogue warp has the result.  `bytes`
  * must cover the slots;
  * pass NULL to stop.  Host-side state, per process.
  */

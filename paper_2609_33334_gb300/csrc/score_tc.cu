@@ -92,9 +92,9 @@ struct TcArgs {
 // CTA at the end into trace[slot * DGE_TRACE_LEN + blockIdx.x].
 enum TraceSlot {
     kTrMmaWaitQ = 0, kTrMmaWaitK, kTrMmaWaitAcc, kTrMmaIssue, kTrMmaCommit, kTrMmaTotal,
-    kTrProdWaitQ, kTrProdWaitK, kTrProdTotal, kTrEpiWaitAcc, kTrStepTimeline, kTrEpiP1End,
-    kTrEpiP2Start, kTrTimeline, kTrEpiTotal, kTrTiles, kTrUnused16, kTrEpiMath, kTrEpiXch,
-    kTrEpiRelease
+    kTrProdWaitQ, kTrProdWaitK, kTrProdTotal, kTrEpiWaitAcc, kTrEpiMathP2, kTrEpiP1End,
+    kTrEpiP2Start, kTrTimeline, kTrEpiTotal, kTrTiles, kTrTileIssue, kTrEpiMath, kTrEpiXch,
+    kTrEpiRelease, kTrTileKReady, kTrTileAccFree, kTrTileIssued, kTrTileEpi
 };
 
 template <bool kTr>
@@ -112,14 +112,6 @@ __device__ __forceinline__ void trace_at(const TcArgs &a, int slot, int i)
         a.trace[slot * DGE_TRACE_LEN + i] = ptx::globaltimer();
 }
 
-// Step timeline of every CTA: global-timer stamp of its phase-1 task i at i * grid + cta.
-template <bool kTr>
-__device__ __forceinline__ void trace_step(const TcArgs &a, int slot, int i)
-{
-    const int64_t idx = (int64_t)i * gridDim.x + blockIdx.x;
-    if (kTr && a.trace && idx < DGE_TRACE_LEN)
-        a.trace[slot * DGE_TRACE_LEN + idx] = ptx::globaltimer();
-}
 
 // SM clock for the cycle accounting; a constant 0 in the kernel built without it.
 template <bool kTr>
@@ -449,7 +441,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             // marks them first to go.
             const uint64_t keep = ptx::make_policy_evict_last();
             const uint64_t drop = ptx::make_policy_evict_first();
-            int ks = 0, qb = 0;
+            int ks = 0, qb = 0, ptc = 0;
             uint32_t kph = 0, qph = 0;
             long long cy_wq = 0, cy_wk = 0;
             const long long cy0 = tclock<kTr>();
@@ -485,6 +477,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                             break;
                         }
                         cy_wk += tclock<kTr>() - c0;
+                        trace_at<kTr>(a, kTrTileIssue, ptc++);
                         ptx::mbar_arrive_expect_tx(&sm.bar[kBarKFull + ks],
                                                    (uint32_t)a.nslab * kSlabBytes);
                         flag[kFlagKArm + ks] = (int)kph;
@@ -534,10 +527,12 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         }
                         long long c1 = tclock<kTr>();
                         cy_wk += c1 - c0;
+                        trace_at<kTr>(a, kTrTileKReady, (int)tc);
                         if (!wait_bar(&sm.bar[kBarAccEmpty + ab], aph ^ 1, flag, a)) {
                             ok = false;
                             break;
                         }
+                        trace_at<kTr>(a, kTrTileAccFree, (int)tc);
                         c0 = tclock<kTr>();
                         cy_wa += c0 - c1;
                         ptx::tc_fence_after();
@@ -563,6 +558,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         ptx::mma_commit(&sm.bar[kBarKEmpty + ks]);
                         ptx::mma_commit(&sm.bar[kBarAccFull + ab]);
                         cy_cm += tclock<kTr>() - c1;
+                        trace_at<kTr>(a, kTrTileIssued, (int)tc);
                         if (++ks == a.kstages) {
                             ks = 0;
                             kph ^= 1;
@@ -728,7 +724,6 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         atomicAdd(&a.count[T.u], 1u);
                     }
                     ptx::mbar_arrive(&sm.bar[kBarRedEmpty + rb]);
-                    trace_step<kTr>(a, kTrStepTimeline, p1c - 1);
                 }
             }
         }
@@ -753,7 +748,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         int p2c = 0;  // phase-2 tasks (-lse buffer p2c % 2)
         bool dead = false;
 
-        long long cy_wa = 0, cy_p1e = 0, cy_p2s = 0, cy_math = 0, cy_xch = 0, cy_rel = 0;
+        long long cy_wa = 0, cy_p1e = 0, cy_p2s = 0, cy_math = 0, cy_math2 = 0, cy_xch = 0, cy_rel = 0;
         const long long cy0 = tclock<kTr>();
         // Waits for this thread's accumulator and returns false once the CTA is dead
         // (the outcome is warp-uniform: the TMEM loads after it are warp-collective).
@@ -766,6 +761,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             if (!dead)
                 ptx::tc_fence_after();
             cy_wa += tclock<kTr>() - c0;
+            if (ew == 0 && lane == 0)
+                trace_at<kTr>(a, kTrTileEpi, tc);
             return !dead;
         };
         // A bounded, warp-uniform wait on a CTA barrier (false once the CTA is dead).
@@ -912,7 +909,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                                         col_add(acc, v, nL[gj], s2, causal, key, first_causal,
                                                 col_base + gj * 16, g.m);
                             });
-                            cy_math += tclock<kTr>() - c0;
+                            cy_math2 += tclock<kTr>() - c0;
                         }
                         // The three warps of this lane quarter (one per warpgroup) leave their
                         // partial sums in shared memory; whichever comes last adds them in
@@ -951,6 +948,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             trace_put<kTr>(a, kTrEpiP1End, cy_p1e);
             trace_put<kTr>(a, kTrEpiP2Start, cy_p2s);
             trace_put<kTr>(a, kTrEpiMath, cy_math);
+            trace_put<kTr>(a, kTrEpiMathP2, cy_math2);
             trace_put<kTr>(a, kTrEpiXch, cy_xch);
             trace_put<kTr>(a, kTrEpiRelease, cy_rel);
             trace_put<kTr>(a, kTrEpiTotal, tclock<kTr>() - cy0);
@@ -1049,7 +1047,23 @@ TcPlan tc_plan(const Geometry &g)
     p.r_pad = (g.R + 15) & ~15;
     p.r4 = (g.R + 3) & ~3;
     p.nslab = g.d / 64;
-    p.chunk_keys = 1024;
+    // Key chunk (one task): as long as the phase-1 data of the tasks between an item's two
+    // phases still fits in L2, i.e. (S + nchunks) chunks of K rows <= L2, which is about
+    // chunk <= (L2 / row_bytes - n) / S.  Longer tasks load the query block less often and
+    // pay the per-task hand-offs less often; measured on GB300 at 32K keys, 24 tiles
+    // (3072 keys) ran 11% faster than 8 and a 32-tile chunk lost L2 hits.  Rounded to a
+    // multiple of 8 tiles, within 8 .. 32 tiles.
+    int dev = 0, l2 = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        sms <= 0)
+        l2 = 0, sms = 1;
+    const double row_bytes = (double)g.d * 2.0;
+    double fit = ((double)l2 / row_bytes - (double)g.n) / (double)sms / kTile;
+    int tiles = (int)(fit / 8.0 + 0.5) * 8;
+    tiles = tiles < 8 ? 8 : (tiles > 32 ? 32 : tiles);
+    p.chunk_keys = tiles * kTile;
     p.nchunks = (g.n + p.chunk_keys - 1) / p.chunk_keys;
     p.kstages = kMaxKStages;
     while (p.kstages > 2 && smem_bytes(p.r_pad, p.nslab, p.kstages) > 232448)
