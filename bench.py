@@ -113,6 +113,8 @@ def kernel_bytes(wl, name):
         return 4 * rows * row_bytes              # K, V rows read + Kc, Vc written
     if name == "select":
         return U * P * 4 + rows * 4              # scores read + idx written
+    if name == "pool_select":
+        return U * P * 4 + rows * 4              # raw scores read + idx written
     if name == "pool":
         return 2 * U * P * 4
     if name == "combine_lse":

@@ -469,7 +469,10 @@ int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
         return rc;
     float *raw = ws_at<float>(ws, plan.off_raw);
     const float *sel = raw;
-    if (g.pool != DGE_POOL_NONE) {
+    if (pool_select_supported(g)) {
+        DGE_LAUNCH("pool_select", stream,
+                   launch_pool_select(g, plan.layers, raw, bufs->scores, bufs->idx, stream));
+    } else if (g.pool != DGE_POOL_NONE) {
         float *pooled = bufs->scores ? bufs->scores : ws_at<float>(ws, plan.off_pooled);
         DGE_LAUNCH("pool", stream, launch_pool(raw, pooled, g.U, g.P, g.pool, g.pool_kernel, stream));
         sel = pooled;
@@ -478,7 +481,8 @@ int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
                                        cudaMemcpyDeviceToDevice, stream),
                        "scores copy");
     }
-    DGE_LAUNCH("select", stream, launch_select(g, plan.layers, sel, bufs->idx, stream));
+    if (!pool_select_supported(g))
+        DGE_LAUNCH("select", stream, launch_select(g, plan.layers, sel, bufs->idx, stream));
     DGE_LAUNCH("compact", stream, launch_compact(g, plan.layers, bufs->idx, nullptr, K, V, bufs->Kc, bufs->Vc,
                                   false, static_cast<uint32_t *>(ws), stream));
     return DGE_OK;

@@ -47,6 +47,11 @@ cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const G
 // Pooling, selection, gather (select_compact.cu).
 cudaError_t launch_pool(const float *raw, float *out, int64_t U, int P, int pool, int kernel,
                         cudaStream_t stream);
+// Pooling and selection in one kernel (the evict path), for P <= 32768 positions per unit.
+// pooled_out (nullable) receives the pooled scores.
+bool pool_select_supported(const Geometry &g);
+cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, const float *raw,
+                               float *pooled_out, int32_t *idx, cudaStream_t stream);
 cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const float *scores,
                           int32_t *idx, cudaStream_t stream);
 cudaError_t launch_streaming_indices(const Geometry &g, const LayerTable &layers, int32_t *idx,

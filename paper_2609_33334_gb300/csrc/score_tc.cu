@@ -71,7 +71,7 @@ struct TcArgs {
     Geometry g;
     int r_pad, r4, nslab, kstages;
     int acc_stride;    // TMEM columns between accumulator buffers
-    int chunk_keys, nchunks;
+    int unit_tiles, nchunks;   // key tiles of a unit; chunk c = tiles [c*T/nc, (c+1)*T/nc)
     int64_t items;
     int64_t lag;       // extra items between an item's phase-1 and phase-2 tasks
     int ng[kEpiWG];    // 16-column groups of each epilogue warpgroup
@@ -147,9 +147,10 @@ __device__ __forceinline__ bool get_task(const TcArgs &a, int64_t t, int j, Task
         return false;
     T.u = item / a.nchunks;
     T.chunk = (int)(item % a.nchunks);
-    T.k_lo = T.chunk * a.chunk_keys;
+    T.k_lo = (int)((int64_t)T.chunk * a.unit_tiles / a.nchunks) * kTile;
+    const int k_end = (int)((int64_t)(T.chunk + 1) * a.unit_tiles / a.nchunks) * kTile;
     const int end = T.phase == 1 ? a.g.n : a.g.P;
-    T.k_hi = min(T.k_lo + a.chunk_keys, end);
+    T.k_hi = min(k_end, end);
     if (T.k_lo >= T.k_hi)
         return false;
     T.ntiles = (T.k_hi - T.k_lo + kTile - 1) / kTile;
@@ -1065,6 +1066,7 @@ TcPlan tc_plan(const Geometry &g)
     tiles = tiles < 8 ? 8 : (tiles > 32 ? 32 : tiles);
     p.chunk_keys = tiles * kTile;
     p.nchunks = (g.n + p.chunk_keys - 1) / p.chunk_keys;
+
     p.kstages = kMaxKStages;
     while (p.kstages > 2 && smem_bytes(p.r_pad, p.nslab, p.kstages) > 232448)
         --p.kstages;
@@ -1099,7 +1101,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.acc_stride = (plan.r_pad + 31) & ~31;
     a.nslab = plan.nslab;
     a.kstages = plan.kstages;
-    a.chunk_keys = plan.chunk_keys;
+    a.unit_tiles = (g.n + kTile - 1) / kTile;
     a.nchunks = plan.nchunks;
     a.items = g.U * plan.nchunks;
     const int NG = plan.r_pad / 16;

@@ -21,6 +21,7 @@ __global__ void pool_kernel(const float *__restrict__ raw, float *__restrict__ o
 {
     const int64_t total = U * (int64_t)P;
     const int r = kernel / 2;
+    const float inv_kernel = 1.0f / (float)kernel;  // avg-pool: in-range sum times 1/K
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t u = i / P;
@@ -40,7 +41,7 @@ __global__ void pool_kernel(const float *__restrict__ raw, float *__restrict__ o
             float s = 0.f;
             for (int q = lo; q <= hi; ++q)
                 s += row[q];
-            out[i] = s / (float)kernel;
+            out[i] = s * inv_kernel;
         }
     }
 }
@@ -233,6 +234,240 @@ cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const flo
     } else {
         select_kernel<false><<<(unsigned)g.U, kSelThreads, 0, stream>>>(scores, idx, p);
     }
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Pooling and selection fused (the evict path, P <= kPsMaxP): one CTA per unit loads the
+// unit's raw scores into shared memory once, pools them (the same arithmetic and order as
+// pool_kernel, so the pooled values are bit-identical), optionally writes them out, and
+// selects from the shared-memory copy.  The kernel is bound by instruction issue, so the
+// radix select takes three passes (11, 11 and 10 bits) and the position-ordered compaction
+// two: a warp's count of kept candidates follows from its counts of keys above and equal to
+// the threshold and the equal keys before it.
+
+constexpr int kPsThreads = 1024;
+constexpr int kPsPer = 32;                       // positions pooled per thread (registers)
+constexpr int kPsMaxP = kPsThreads * kPsPer;     // 32768
+constexpr int kPsBins = 2048;                    // radix bins (11 bits)
+
+// Exclusive scan of one int per warp (cnt[0..kSelWarps)) into base[], by warp 0.
+__device__ __forceinline__ void scan_warp_counts(const int *cnt, int *base)
+{
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        const int v = lane < kSelWarps ? cnt[lane] : 0;
+        int incl = v;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int o = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off)
+                incl += o;
+        }
+        if (lane < kSelWarps)
+            base[lane] = incl - v;
+    }
+}
+
+// Pooled value at position j of a row of P raw scores in shared memory.  R > 0: the pool
+// radius known at compile time (interior positions unrolled); R < 0: radius r at run time.
+template <int POOL, int R>
+__device__ __forceinline__ float pool_at(const float *sraw, int j, int P, int r, int kernel)
+{
+    if (POOL == DGE_POOL_NONE)
+        return sraw[j];
+    const int rr = R > 0 ? R : r;
+    const int lo = max(0, j - rr), hi = min(P - 1, j + rr);
+    float x = POOL == DGE_POOL_MAX ? -INFINITY : 0.f;
+    if (R > 0 && j >= R && j + R < P) {
+#pragma unroll
+        for (int q = -R; q <= R; ++q)
+            x = POOL == DGE_POOL_MAX ? fmaxf(x, sraw[j + q]) : x + sraw[j + q];
+    } else {
+        for (int q = lo; q <= hi; ++q)
+            x = POOL == DGE_POOL_MAX ? fmaxf(x, sraw[q]) : x + sraw[q];
+    }
+    return POOL == DGE_POOL_AVG ? x * (1.0f / (float)kernel) : x;
+}
+
+template <int POOL, int R>
+__global__ void __launch_bounds__(kPsThreads, 1)
+pool_select_kernel(const float *__restrict__ raw, float *__restrict__ pooled_out,
+                   int32_t *__restrict__ idx, SelectParams p, int kernel)
+{
+    extern __shared__ __align__(16) uint32_t sbuf[];  // [P]: raw scores, then pooled keys
+    __shared__ uint32_t hist[kPsBins];
+    __shared__ int warp_cnt[kSelWarps], warp_base[kSelWarps], warp_gt[kSelWarps];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_rank;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint32_t lt_mask = (1u << lane) - 1u;
+    const int64_t u = blockIdx.x;
+    const Geometry &g = p.g;
+    int budget;
+    int32_t *out = idx + unit_row_base(p, u, budget);
+    const int P = g.P, s0 = g.sinks, tail = g.n - g.P;
+    const int C = P - s0;                    // candidates [s0, P)
+    const int keep = budget - s0 - tail;     // candidates to keep
+
+    // Raw scores to shared memory, pooled values to registers, then keys in place.
+    const float *row = raw + u * (int64_t)P;
+    float *sraw = reinterpret_cast<float *>(sbuf);
+    for (int j = tid; j < P; j += kPsThreads)
+        sraw[j] = row[j];
+    __syncthreads();
+    float v[kPsPer];
+#pragma unroll
+    for (int i = 0; i < kPsPer; ++i) {
+        const int j = tid + i * kPsThreads;
+        v[i] = j < P ? pool_at<POOL, R>(sraw, j, P, kernel / 2, kernel) : 0.f;
+    }
+    __syncthreads();
+    float *pout = pooled_out ? pooled_out + u * (int64_t)P : nullptr;
+#pragma unroll
+    for (int i = 0; i < kPsPer; ++i) {
+        const int j = tid + i * kPsThreads;
+        if (j < P) {
+            if (pout)
+                pout[j] = v[i];
+            sbuf[j] = float_key(v[i]);
+        }
+    }
+    __syncthreads();
+
+    for (int j = tid; j < s0; j += kPsThreads)
+        out[j] = j;
+    for (int j = tid; j < tail; j += kPsThreads)
+        out[s0 + keep + j] = P + j;
+    if (keep <= 0)
+        return;
+    if (keep >= C) {
+        for (int j = tid; j < C; j += kPsThreads)
+            out[s0 + j] = s0 + j;
+        return;
+    }
+    const uint32_t *keys = sbuf + s0;
+
+    // Radix select from the top, 11 + 11 + 10 bits: T = the keep-th largest key.
+    uint32_t prefix = 0, mask = 0;
+    int rank = keep;
+#pragma unroll 1
+    for (int pass = 0; pass < 3; ++pass) {
+        const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
+        const uint32_t bmask = pass == 2 ? 1023u : 2047u;
+        for (int i = tid; i < kPsBins; i += kPsThreads)
+            hist[i] = 0;
+        __syncthreads();
+        for (int j = tid; j < C; j += kPsThreads) {
+            const uint32_t k = keys[j];
+            if ((k & mask) == prefix)
+                atomicAdd(&hist[(k >> shift) & bmask], 1u);
+        }
+        __syncthreads();
+        if (tid < 32) {
+            // Suffix counts over the bins, from the top: lane handles 64 consecutive bins.
+            const int nb = (int)bmask + 1, per = nb / 32;
+            const int top = nb - 1 - lane * per;   // this lane's bins: top, top-1, ...
+            uint32_t local = 0;
+            for (int q = 0; q < per; ++q)
+                local += hist[top - q];
+            uint32_t incl = local;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const uint32_t o = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off)
+                    incl += o;
+            }
+            uint32_t run = incl - local;
+            if (run < (uint32_t)rank && run + local >= (uint32_t)rank) {
+                for (int q = 0; q < per; ++q) {
+                    const uint32_t c = hist[top - q];
+                    if (run + c >= (uint32_t)rank) {
+                        s_prefix = prefix | ((uint32_t)(top - q) << shift);
+                        s_rank = rank - (int)run;
+                        break;
+                    }
+                    run += c;
+                }
+            }
+        }
+        __syncthreads();
+        prefix = s_prefix;
+        rank = s_rank;
+        mask |= bmask << shift;
+        __syncthreads();
+    }
+    const uint32_t T = prefix;
+    const int need_eq = rank;  // keys equal to T to keep, lowest positions first
+
+    // Position-ordered compaction: warp w owns candidates [w_lo, w_hi).  Pass 1 counts the
+    // keys above and equal to T; the warp keeps its keys above T and the equal keys whose
+    // rank among all equal keys is below need_eq.
+    const int per_w = ((C + kSelWarps - 1) / kSelWarps + 31) & ~31;
+    const int w_lo = min(C, warp * per_w), w_hi = min(C, w_lo + per_w);
+    int eq_cnt = 0, gt_cnt = 0;
+    for (int c = w_lo; c < w_hi; c += 32) {
+        const int j = c + lane;
+        const uint32_t k = j < w_hi ? keys[j] : 0u;
+        eq_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k == T));
+        gt_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k > T));
+    }
+    if (lane == 0) {
+        warp_cnt[warp] = eq_cnt;
+        warp_gt[warp] = gt_cnt;
+    }
+    __syncthreads();
+    scan_warp_counts(warp_cnt, warp_base);
+    __syncthreads();
+    const int eq_base = warp_base[warp];
+    const int eq_kept = min(eq_cnt, max(0, need_eq - eq_base));
+    __syncthreads();                      // every warp has read its equal-key offset
+    if (lane == 0)
+        warp_cnt[warp] = warp_gt[warp] + eq_kept;
+    __syncthreads();
+    scan_warp_counts(warp_cnt, warp_base);
+    __syncthreads();
+    int sel_run = warp_base[warp], eq_run = eq_base;
+    for (int c = w_lo; c < w_hi; c += 32) {
+        const int j = c + lane;
+        const uint32_t k = j < w_hi ? keys[j] : 0u;
+        const bool eq = j < w_hi && k == T;
+        const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+        const bool sel = j < w_hi && (k > T || (eq && eq_run + __popc(eqb & lt_mask) < need_eq));
+        const uint32_t selb = __ballot_sync(0xffffffffu, sel);
+        const int pos = sel_run + __popc(selb & lt_mask);
+        if (sel && pos < keep)
+            out[s0 + pos] = s0 + j;
+        sel_run += __popc(selb);
+        eq_run += __popc(eqb);
+    }
+}
+
+bool pool_select_supported(const Geometry &g) { return g.P <= kPsMaxP; }
+
+cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, const float *raw,
+                               float *pooled_out, int32_t *idx, cudaStream_t stream)
+{
+    SelectParams p;
+    p.g = g;
+    p.layers = layers;
+    const size_t smem = (size_t)max(g.P, 1) * sizeof(uint32_t);
+    using KernT = void (*)(const float *, float *, int32_t *, SelectParams, int);
+    KernT kern;
+    if (g.pool == DGE_POOL_MAX)
+        kern = g.pool_kernel == 7 ? pool_select_kernel<DGE_POOL_MAX, 3>
+                                  : pool_select_kernel<DGE_POOL_MAX, -1>;
+    else if (g.pool == DGE_POOL_AVG)
+        kern = g.pool_kernel == 7 ? pool_select_kernel<DGE_POOL_AVG, 3>
+                                  : pool_select_kernel<DGE_POOL_AVG, -1>;
+    else
+        kern = pool_select_kernel<DGE_POOL_NONE, 0>;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem);
+    if (err != cudaSuccess)
+        return err;
+    kern<<<(unsigned)g.U, kPsThreads, smem, stream>>>(raw, pooled_out, idx, p, g.pool_kernel);
     return cudaGetLastError();
 }
 

@@ -67,6 +67,7 @@ SMALL = {
     "short_cache": WL["c1_tiny"].with_(n=37, budgets=(20,), n_spans=0),
     "sinks_scored": WL["c1_tiny"].with_(sinks=4, budgets=(100,)),
     "no_pool": WL["c1_tiny"].with_(pool=inputs.POOL_NONE, pool_kernel=1),
+    "long_p": WL["c1_tiny"].with_(n=33500, budgets=(600,), n_spans=0),  # P > 32768
     "avg_pool_31": WL["c1_tiny"].with_(pool=inputs.POOL_AVG, pool_kernel=31),
     "max_pool_3_d128": WL["c1_tiny"].with_(d=128, pool_kernel=3),
     "gqa8_ragged": WL["c1_tiny"].with_(Hq=16, Hkv=2, n=2117, budgets=(333,)),
@@ -111,9 +112,15 @@ def test_runs_are_bit_identical():
         assert torch.equal(a[k], b[k]), k
 
 
-def test_separate_calls_match_fused():
-    """dge_score -> dge_select -> dge_compact equals dge_evict."""
-    wl = SMALL["c2_small"]
+@pytest.mark.parametrize("name", ["c2_small", "c3_small", "no_pool", "keep_none", "keep_all",
+                                  "long_p"])
+def test_separate_calls_match_fused(name):
+    """dge_score -> dge_select -> dge_compact equals dge_evict, bit for bit.
+
+    dge_evict pools and selects in one kernel (P <= 32768) while the separate calls run the
+    pooling and selection kernels; max-, avg- and no pooling, the degenerate budgets, and a
+    case through the larger-P path."""
+    wl = SMALL[name]
     tens, fused = run(wl)
     p = api.problem_from_workload(wl)
     s = api.score(p, tens["K"], tens["Q"])
