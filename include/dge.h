@@ -110,6 +110,19 @@ typedef struct dge_buffers {
     int32_t *idx;        /* packed kept positions (dge_evict) */
     void *Kc;            /* packed [rows][d] bf16 (dge_evict) */
     void *Vc;            /* packed [rows][d] bf16 (dge_evict) */
+    /* Row normalisers, fp32, natural log, dense [L][b][Hq][rows] (rows = m for SCORED, n for
+     * H2O), row i of query head h at position pos_i:
+     *   lse[l][b][h][i] = log sum_{j <= pos_i} exp(scale * q . k_j)   (scale as in the problem).
+     * lse_in (optional): supplied by the caller -- the attention pass that produced the draft
+     * (or window) rows already forms this normaliser (flash attention returns it), which is
+     * why the paper counts the draft's scores as free (Sec. "Draft-Guided Eviction", phase B;
+     * App. "Complexity and overheads").  With lse_in the scoring skips its normaliser pass
+     * and reads K once.  The caller vouches for the values: they must be finite, and scores
+     * are exp(s - lse) summed as given.
+     * lse_out (optional, ignored when lse_in is set): receives the normalisers the scoring
+     * computed.  Both 4-byte aligned; NULL to leave unused. */
+    const float *lse_in;
+    float *lse_out;
 } dge_buffers;
 
 /*

@@ -49,6 +49,12 @@ class Problem:
     def packed_rows(self) -> int:
         return B.dge_packed_rows(self.c())
 
+    @property
+    def lse_shape(self) -> tuple:
+        """Layout of the row normalisers (dge_buffers.lse_in / lse_out): [L][b][Hq][rows]."""
+        rows = self.n if self.variant == B.DGE_VARIANT_H2O else self.m
+        return (self.L, self.b, self.Hq, rows)
+
     def workspace_bytes(self) -> int:
         return B.dge_workspace_size(self.c())
 
@@ -87,12 +93,24 @@ def _check_cache(t: torch.Tensor, name: str) -> None:
         raise ValueError(f"{name} must be a bf16 CUDA tensor")
 
 
+def _lse_arg(p: Problem, lse_in: Optional[torch.Tensor]) -> int:
+    if lse_in is None:
+        return 0
+    if lse_in.dtype != torch.float32 or not lse_in.is_contiguous() or \
+            tuple(lse_in.shape) != p.lse_shape:
+        raise ValueError(f"lse_in must be contiguous float32 of shape {p.lse_shape}")
+    return lse_in.data_ptr()
+
+
 def evict(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torch.Tensor] = None, *,
-          want_scores: bool = False, ws: Optional[torch.Tensor] = None,
+          want_scores: bool = False, lse_in: Optional[torch.Tensor] = None,
+          want_lse: bool = False, ws: Optional[torch.Tensor] = None,
           out: Optional[dict] = None, stream=None) -> dict:
     """dge_evict: the fused score -> pool -> select -> compact pass.
 
-    Returns {"idx", "Kc", "Vc", "scores"} (scores is None unless requested).
+    Returns {"idx", "Kc", "Vc", "scores", "lse"} (scores / lse are None unless requested).
+    ``lse_in``: the rows' natural-log normalisers [L][b][Hq][rows] (Problem.lse_shape), so the
+    scoring reads K once; ``want_lse``: return the normalisers the scoring computed.
     ``out`` may hold preallocated outputs with those keys.
     """
     _check_cache(K, "K")
@@ -109,25 +127,35 @@ def evict(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torch.Tensor
     if want_scores and o.get("scores") is None:
         o["scores"] = torch.empty((p.U, p.P), dtype=torch.float32, device=dev)
     o.setdefault("scores", None)
+    if want_lse and lse_in is None and o.get("lse") is None:
+        o["lse"] = torch.empty(p.lse_shape, dtype=torch.float32, device=dev)
+    o.setdefault("lse", None)
     if ws is None:
         ws = workspace(p, dev)
     bufs = B.dge_buffers(K=B.tensor_desc(K), V=B.tensor_desc(V), Q=B.tensor_desc(Q),
                          scores=B.ptr(o["scores"]), idx=B.ptr(o["idx"]), Kc=B.ptr(o["Kc"]),
-                         Vc=B.ptr(o["Vc"]))
+                         Vc=B.ptr(o["Vc"]), lse_in=_lse_arg(p, lse_in),
+                         lse_out=B.ptr(o["lse"]) if want_lse and lse_in is None else 0)
     B.dge_evict(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
     return o
 
 
-def score(p: Problem, K: torch.Tensor, Q: torch.Tensor, *, ws=None, stream=None) -> torch.Tensor:
-    """dge_score: final (pooled) scores [unit][P] in float32."""
+def score(p: Problem, K: torch.Tensor, Q: torch.Tensor, *, lse_in=None, want_lse=False,
+          ws=None, stream=None):
+    """dge_score: final (pooled) scores [unit][P] in float32.
+
+    With ``want_lse`` returns (scores, lse); ``lse_in`` as for evict()."""
     _check_cache(K, "K")
     _check_cache(Q, "Q")
     scores = torch.empty((p.U, p.P), dtype=torch.float32, device=K.device)
+    lse = torch.empty(p.lse_shape, dtype=torch.float32, device=K.device) \
+        if want_lse and lse_in is None else None
     if ws is None:
         ws = workspace(p, K.device)
-    bufs = B.dge_buffers(K=B.tensor_desc(K), Q=B.tensor_desc(Q), scores=scores.data_ptr())
+    bufs = B.dge_buffers(K=B.tensor_desc(K), Q=B.tensor_desc(Q), scores=scores.data_ptr(),
+                         lse_in=_lse_arg(p, lse_in), lse_out=B.ptr(lse))
     B.dge_score(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
-    return scores
+    return (scores, lse) if want_lse else scores
 
 
 def select(p: Problem, scores: Optional[torch.Tensor], *, stream=None) -> torch.Tensor:

@@ -40,7 +40,8 @@ class dge_tensor(ctypes.Structure):
 
 class dge_buffers(ctypes.Structure):
     _fields_ = [("K", dge_tensor), ("V", dge_tensor), ("Q", dge_tensor), ("scores", c_void_p),
-                ("idx", c_void_p), ("Kc", c_void_p), ("Vc", c_void_p)]
+                ("idx", c_void_p), ("Kc", c_void_p), ("Vc", c_void_p), ("lse_in", c_void_p),
+                ("lse_out", c_void_p)]
 
 
 class dge_kernel_time(ctypes.Structure):

@@ -293,14 +293,40 @@ bool want_tc(const Geometry &g)
     return tc_supported(g);
 }
 
-// raw scores of every unit into the workspace.
+// raw scores of every unit into the workspace.  lse_in (nullable): the caller's natural-log
+// row normalisers, so only the column-sum pass runs; lse_out (nullable, ignored with lse_in):
+// receives the normalisers computed here.
 int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void *ws,
-                cudaStream_t stream)
+                cudaStream_t stream, const float *lse_in, float *lse_out)
 {
     const Geometry &g = plan.g;
     float2 *partial = ws_at<float2>(ws, plan.off_partial);
     float *lse2 = ws_at<float>(ws, plan.off_lse);
     float *raw = ws_at<float>(ws, plan.off_raw);
+    if (lse_in) {
+        if (g.variant == DGE_VARIANT_SCORED && want_tc(g)) {
+            TcBuffers tb;
+            tb.part = nullptr;
+            tb.lse2 = lse2;
+            tb.raw = raw;
+            tb.count = nullptr;
+            tb.ready = nullptr;
+            tb.status = static_cast<uint32_t *>(ws);
+            tb.lse_in = lse_in;
+            bool encoded = false;
+            DGE_LAUNCH("score_tc_lse", stream,
+                       launch_score_tc(K, Q, g, plan.tc, tb, stream, &encoded));
+            if (encoded)
+                return DGE_OK;
+        }
+        DGE_LAUNCH("lse_import", stream, launch_lse_import(lse_in, lse2, g.U * g.R, stream));
+        if (g.variant == DGE_VARIANT_H2O)
+            DGE_LAUNCH("colsum_keys", stream, launch_colsum_keys(K, Q, g, lse2, raw, stream));
+        else
+            DGE_LAUNCH("colsum_rows", stream,
+                       launch_colsum_rows(K, Q, g, kScoredChunkKeys, lse2, raw, stream));
+        return DGE_OK;
+    }
     if (g.variant == DGE_VARIANT_SCORED && want_tc(g)) {
         uint32_t *count = ws_at<uint32_t>(ws, plan.off_count);
         uint32_t *ready = ws_at<uint32_t>(ws, plan.off_ready);
@@ -327,6 +353,10 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
                        launch_combine_lse(partial, g.U * g.R, 1, lse2, stream, ready, g.R));
             DGE_LAUNCH("recompute_colsum", stream,
                        launch_colsum_rows(K, Q, g, g.P, lse2, raw, stream, ready));
+            if (lse_out)
+                DGE_LAUNCH("lse_export", stream,
+                           launch_lse_export(tb.part, plan.tc.nchunks, plan.tc.r4, lse2, ready,
+                                             g.U, g.R, lse_out, stream));
             return DGE_OK;
         }
     }
@@ -337,7 +367,16 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
         DGE_LAUNCH("colsum_keys", stream, launch_colsum_keys(K, Q, g, lse2, raw, stream));
     else
         DGE_LAUNCH("colsum_rows", stream, launch_colsum_rows(K, Q, g, kScoredChunkKeys, lse2, raw, stream));
+    if (lse_out)
+        DGE_LAUNCH("lse_export", stream,
+                   launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, lse_out, stream));
     return DGE_OK;
+}
+
+// Row normaliser pointers: 4-byte aligned or NULL.
+bool lse_ptrs_ok(const dge_buffers *bufs)
+{
+    return ((uintptr_t)bufs->lse_in & 3) == 0 && ((uintptr_t)bufs->lse_out & 3) == 0;
 }
 
 }  // namespace
@@ -385,11 +424,12 @@ int dge_score(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
     if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->Q)) != DGE_OK ||
         (rc = check_ws(plan, ws, ws_bytes)) != DGE_OK)
         return rc;
-    if (((uintptr_t)bufs->scores & 3) != 0)
+    if (((uintptr_t)bufs->scores & 3) != 0 || !lse_ptrs_ok(bufs))
         return DGE_ERR_UNSUPPORTED;
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
     DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
-    if ((rc = run_scoring(plan, desc(bufs->K), desc(bufs->Q), ws, stream)) != DGE_OK)
+    if ((rc = run_scoring(plan, desc(bufs->K), desc(bufs->Q), ws, stream, bufs->lse_in,
+                          bufs->lse_out)) != DGE_OK)
         return rc;
     DGE_LAUNCH("pool", stream, launch_pool(ws_at<float>(ws, plan.off_raw), bufs->scores, plan.g.U, plan.g.P,
                                plan.g.pool, plan.g.pool_kernel, stream));
@@ -447,7 +487,7 @@ int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
     if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK)
         return rc;
     if (((uintptr_t)bufs->Kc & 15) || ((uintptr_t)bufs->Vc & 15) || ((uintptr_t)bufs->idx & 3) ||
-        ((uintptr_t)bufs->scores & 3))
+        ((uintptr_t)bufs->scores & 3) || !lse_ptrs_ok(bufs))
         return DGE_ERR_UNSUPPORTED;
     const Geometry &g = plan.g;
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
@@ -465,7 +505,7 @@ int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
         return rc;
     DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
     const TensorDesc K = desc(bufs->K), V = desc(bufs->V), Q = desc(bufs->Q);
-    if ((rc = run_scoring(plan, K, Q, ws, stream)) != DGE_OK)
+    if ((rc = run_scoring(plan, K, Q, ws, stream, bufs->lse_in, bufs->lse_out)) != DGE_OK)
         return rc;
     float *raw = ws_at<float>(ws, plan.off_raw);
     const float *sel = raw;

@@ -29,8 +29,9 @@ struct TcBuffers {
     float *lse2;       // [U][R]
     float *raw;        // [U][P]
     uint32_t *count;   // [U], zero before the launch
-    uint32_t *ready;   // [U], zero before the launch; 1 = lse ready, 2 = recompute
+    uint32_t *ready;   // [U], zero before the launch; 2 = recompute
     uint32_t *status;
+    const float *lse_in = nullptr;  // [U][R] supplied natural-log normalisers (one pass)
 };
 bool tc_supported(const Geometry &g);
 // Trace buffer of the tensor-core scoring kernel (see dge_trace_set); nullptr = off.
@@ -47,6 +48,12 @@ cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const G
 // Pooling, selection, gather (select_compact.cu).
 cudaError_t launch_pool(const float *raw, float *out, int64_t U, int P, int pool, int kernel,
                         cudaStream_t stream);
+// Row normalisers: caller's natural-log [U][R] -> base-2 lse2; lse2 (or, on the tensor-core
+// path, its chunk sums part [U][nchunks][r4] for units with ready != 2) -> natural-log out.
+cudaError_t launch_lse_import(const float *lse_in, float *lse2, int64_t total, cudaStream_t stream);
+cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const float *lse2,
+                              const uint32_t *ready, int64_t U, int R, float *lse_out,
+                              cudaStream_t stream);
 // Pooling and selection in one kernel (the evict path), for P <= 32768 positions per unit.
 // pooled_out (nullable) receives the pooled scores.
 bool pool_select_supported(const Geometry &g);

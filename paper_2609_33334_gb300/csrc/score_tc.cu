@@ -74,6 +74,8 @@ struct TcArgs {
     int unit_tiles, nchunks;   // key tiles of a unit; chunk c = tiles [c*T/nc, (c+1)*T/nc)
     int64_t items;
     int64_t lag;       // extra items between an item's phase-1 and phase-2 tasks
+    const float *lse_in;  // [U][R] natural-log row normalisers supplied by the caller: then
+                          // there is no phase 1 and phase 2 of item t*S + s runs in step t
     int ng[kEpiWG];    // 16-column groups of each epilogue warpgroup
     int gbase[kEpiWG]; // first group of each epilogue warpgroup
     int64_t steps;
@@ -136,7 +138,12 @@ __device__ __forceinline__ bool get_task(const TcArgs &a, int64_t t, int j, Task
 {
     const int64_t S = gridDim.x, s = blockIdx.x;
     int64_t item;
-    if (j == 0) {
+    if (a.lse_in) {
+        if (j == 0)
+            return false;
+        item = t * S + s;
+        T.phase = 2;
+    } else if (j == 0) {
         item = t * S + s;
         T.phase = 1;
     } else {
@@ -631,6 +638,20 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 if (lane == 0)
                     trace_at<kTr>(a, kTrTimeline, 4 * (p2c - 1));
                 int got = wait_w(&sm.bar[kBarLseEmpty + lb], lph ^ 1) ? 1 : 0;
+                if (a.lse_in) {
+                    // Supplied normalisers: -lse in base 2, straight from the caller's array.
+                    float *L = sm.sL + lb * 256;
+                    const float *src = a.lse_in + T.u * g.R;
+                    for (int r = lane; r < a.r_pad; r += 32)
+                        L[r] = (got && r < g.R) ? -__ldg(src + r) * 1.4426950408889634f
+                                                : -INFINITY;
+                    __syncwarp();
+                    if (lane == 0) {
+                        sm.sLbad[lb] = (!got || flag[kFlagAbort]) ? 1 : 0;
+                        ptx::mbar_arrive(&sm.bar[kBarLseFull + lb]);
+                    }
+                    continue;
+                }
                 if (lane == 0) {
                     trace_at<kTr>(a, kTrTimeline, 4 * (p2c - 1) + 1);
                     got = got && spin_count(&a.count[T.u]);
@@ -1103,7 +1124,12 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.kstages = plan.kstages;
     a.unit_tiles = (g.n + kTile - 1) / kTile;
     a.nchunks = plan.nchunks;
-    a.items = g.U * plan.nchunks;
+    a.lse_in = buf.lse_in;
+    if (a.lse_in) {
+        // One pass, nothing to keep in L2: tasks of up to 32 tiles.
+        a.nchunks = (a.unit_tiles + 31) / 32;
+    }
+    a.items = g.U * a.nchunks;
     const int NG = plan.r_pad / 16;
     for (int w = 0, base = 0; w < kEpiWG; ++w) {
         a.ng[w] = NG / kEpiWG + (w < NG % kEpiWG ? 1 : 0);
@@ -1111,7 +1137,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
         base += a.ng[w];
     }
     const int64_t grid = a.items < sms ? a.items : sms;
-    a.lag = plan.nchunks - 1;
+    a.lag = a.lse_in ? 0 : a.nchunks - 1;
     // Phase 2 of the last item runs in step `steps`: (steps - 1) * grid + s - lag covers it.
     a.steps = (a.items + a.lag + grid - 1) / grid;
     a.part = buf.part;

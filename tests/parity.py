@@ -68,9 +68,10 @@ def check_kept(idx: np.ndarray, ref_scores: np.ndarray, ref_idx: np.ndarray, *, 
     return len(diff)
 
 
-def oracle_units(wl, tens, units):
+def oracle_units(wl, tens, units, want_lse=False):
     """Oracle results for several units, the scores of all of them in one
-    multi-threaded oracle call; returns {(l, b, h): evict_unit-style dict}."""
+    multi-threaded oracle call; returns {(l, b, h): evict_unit-style dict} (with the
+    unit's row normalisers [R], natural log, under "lse" when ``want_lse``)."""
     refs = {}
     if wl.variant == inputs.STREAMING:
         for (l, b, h) in units:
@@ -86,12 +87,17 @@ def oracle_units(wl, tens, units):
     K = np.stack([unit_bits(tens["K"], l, b, h) for (l, b, h) in units])
     pos = oracle.h2o_positions(wl.n, G) if wl.variant == inputs.H2O else \
         oracle.scored_positions(wl.n, wl.m, G)
-    raw = oracle.scores(Q, K, pos, wl.n - wl.tail)
+    if want_lse:
+        raw, lse = oracle.scores(Q, K, pos, wl.n - wl.tail, want_lse=True)
+    else:
+        raw, lse = oracle.scores(Q, K, pos, wl.n - wl.tail), None
     for i, (l, b, h) in enumerate(units):
         pooled = oracle.pool(raw[i], wl.pool, wl.pool_kernel) if wl.variant == inputs.SCORED \
             else raw[i].copy()
         idx = oracle.select(pooled, wl.n, wl.sinks, wl.tail, wl.budgets[l])
         refs[(l, b, h)] = {"raw": raw[i], "pooled": pooled, "idx": idx}
+        if lse is not None:
+            refs[(l, b, h)]["lse"] = lse[i]
     return refs
 
 

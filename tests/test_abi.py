@@ -48,7 +48,9 @@ def test_struct_layout_matches_c():
     assert B.dge_problem.seq_len.offset == 24
     assert B.dge_problem.budgets.offset == 56
     assert ctypes.sizeof(B.dge_tensor) == 40
-    assert ctypes.sizeof(B.dge_buffers) == 3 * 40 + 4 * 8
+    assert ctypes.sizeof(B.dge_buffers) == 3 * 40 + 6 * 8
+    assert B.dge_buffers.lse_in.offset == 3 * 40 + 4 * 8
+    assert B.dge_buffers.lse_out.offset == 3 * 40 + 5 * 8
 
 
 def test_pyramid_budgets_paper_examples(lib):
@@ -142,6 +144,17 @@ def test_null_and_misaligned_arguments_rejected_before_launch(lib):
     bufs.scores = 0x5000
     assert lib.dge_score(ctypes.byref(ps), ctypes.byref(bufs), 0x10000, need.value, None) == \
         B.DGE_ERR_INVALID_ARG
+    # misaligned row normalisers (supplied or requested)
+    bufs.lse_in = 0x6002
+    assert lib.dge_score(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value, None) == \
+        B.DGE_ERR_UNSUPPORTED
+    assert lib.dge_evict(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value, None) == \
+        B.DGE_ERR_UNSUPPORTED
+    bufs.lse_in = 0
+    bufs.lse_out = 0x6001
+    assert lib.dge_evict(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value, None) == \
+        B.DGE_ERR_UNSUPPORTED
+    bufs.lse_out = 0
     assert lib.dge_select(ctypes.byref(p), None, 0x2000, None) == B.DGE_ERR_INVALID_ARG
     assert lib.dge_compact(ctypes.byref(p), None, None, None, 0, 0, None, None) == \
         B.DGE_ERR_INVALID_ARG
