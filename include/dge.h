@@ -201,6 +201,28 @@ int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
               void *stream);
 
 /*
+ * In-place compaction (Alg. 1: each head's cache is edited once, in place, temporal order
+ * kept; App. E sorts the kept indices before the gather): rows [0, B_l) of every unit of K
+ * and V become the kept rows, in ascending position order; rows [B_l, n) keep their old
+ * contents.  K->data and V->data are WRITTEN (the cache the caller decodes from next).
+ * idx: packed kept positions as dge_select writes them; each unit's must ascend (then
+ * idx[r] >= r and the forward copy is safe).  A position outside [r, n) is skipped and
+ * reported in the status word of ws (DGE_ERR_INVALID_ARG; like dge_compact, this call does
+ * not clear the word first); ws may be NULL.
+ */
+int dge_compact_inplace(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
+                        const dge_tensor *V, void *ws, void *stream);
+
+/*
+ * dge_evict with the in-place compaction: score -> pool -> select, then the kept rows move
+ * to the front of every unit of bufs->K and bufs->V (their data is WRITTEN).  bufs->Kc and
+ * bufs->Vc are ignored; bufs->idx, scores, lse_in and lse_out as for dge_evict.  The scoring
+ * finishes before the gather starts (same stream), so the scores see the cache as it was.
+ */
+int dge_evict_inplace(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+                      void *stream);
+
+/*
  * PyramidKV's per-layer past budgets (App. L): c = B - w, min = floor(c/20),
  * max = 2c - min, steps = floor((max - min)/(L - 1)), out[l] = max - l*steps.
  * These are past tokens only; add the protected tail to get dge budgets.

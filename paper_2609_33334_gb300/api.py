@@ -180,6 +180,43 @@ def compact(p: Problem, idx: torch.Tensor, K: torch.Tensor, V: torch.Tensor, *, 
     return Kc, Vc
 
 
+def compact_inplace(p: Problem, idx: torch.Tensor, K: torch.Tensor, V: torch.Tensor, *,
+                    ws=None, stream=None) -> None:
+    """dge_compact_inplace: rows [0, B_l) of every unit of K and V become the kept rows."""
+    _check_cache(K, "K")
+    _check_cache(V, "V")
+    B.dge_compact_inplace(p.c(), idx.data_ptr(), B.tensor_desc(K), B.tensor_desc(V),
+                          B.ptr(ws), _stream(stream))
+
+
+def evict_inplace(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torch.Tensor] = None,
+                  *, want_scores: bool = False, lse_in: Optional[torch.Tensor] = None,
+                  want_lse: bool = False, ws: Optional[torch.Tensor] = None,
+                  out: Optional[dict] = None, stream=None) -> dict:
+    """dge_evict_inplace: score -> pool -> select, then the kept rows move to the front of
+    every unit of K and V (written in place).  Returns {"idx", "scores", "lse"}."""
+    _check_cache(K, "K")
+    _check_cache(V, "V")
+    dev = K.device
+    o = dict(out or {})
+    if o.get("idx") is None:
+        o["idx"] = torch.empty(p.packed_rows(), dtype=torch.int32, device=dev)
+    if want_scores and o.get("scores") is None:
+        o["scores"] = torch.empty((p.U, p.P), dtype=torch.float32, device=dev)
+    o.setdefault("scores", None)
+    if want_lse and lse_in is None and o.get("lse") is None:
+        o["lse"] = torch.empty(p.lse_shape, dtype=torch.float32, device=dev)
+    o.setdefault("lse", None)
+    if ws is None:
+        ws = workspace(p, dev)
+    bufs = B.dge_buffers(K=B.tensor_desc(K), V=B.tensor_desc(V), Q=B.tensor_desc(Q),
+                         scores=B.ptr(o["scores"]), idx=B.ptr(o["idx"]),
+                         lse_in=_lse_arg(p, lse_in),
+                         lse_out=B.ptr(o["lse"]) if want_lse and lse_in is None else 0)
+    B.dge_evict_inplace(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
+    return o
+
+
 def device_status(ws: torch.Tensor, stream=None) -> int:
     """dge_get_device_status: sync the stream and read/clear the status word."""
     return B.dge_get_device_status(ws.data_ptr(), _stream(stream))

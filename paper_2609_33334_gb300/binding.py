@@ -71,6 +71,8 @@ _SIGS = {
     "dge_select": [_P, c_void_p, c_void_p, c_void_p],
     "dge_compact": [_P, c_void_p, _T, _T, c_void_p, c_void_p, c_void_p, c_void_p],
     "dge_evict": [_P, _B, c_void_p, c_size_t, c_void_p],
+    "dge_evict_inplace": [_P, _B, c_void_p, c_size_t, c_void_p],
+    "dge_compact_inplace": [_P, c_void_p, _T, _T, c_void_p, c_void_p],
     "dge_pyramid_budgets": [c_int32, c_int32, c_int32, POINTER(c_int32)],
     "dge_get_device_status": [c_void_p, c_void_p],
     "dge_status_string": [c_int],
@@ -141,6 +143,19 @@ def dge_compact(p: dge_problem, idx: int, K: dge_tensor, V: dge_tensor, Kc: int,
                 ws: int, stream: int) -> None:
     _check("dge_compact", _lib().dge_compact(ctypes.byref(p), idx, ctypes.byref(K),
                                              ctypes.byref(V), Kc, Vc, ws, stream))
+
+
+def dge_evict_inplace(p: dge_problem, bufs: dge_buffers, ws: int, ws_bytes: int,
+                      stream: int) -> None:
+    _check("dge_evict_inplace", _lib().dge_evict_inplace(ctypes.byref(p), ctypes.byref(bufs), ws,
+                                                         ws_bytes, stream))
+
+
+def dge_compact_inplace(p: dge_problem, idx: int, K: dge_tensor, V: dge_tensor, ws: int,
+                        stream: int) -> None:
+    _check("dge_compact_inplace", _lib().dge_compact_inplace(ctypes.byref(p), idx,
+                                                             ctypes.byref(K), ctypes.byref(V),
+                                                             ws, stream))
 
 
 def dge_evict(p: dge_problem, bufs: dge_buffers, ws: int, ws_bytes: int, stream: int) -> None:

@@ -475,36 +475,49 @@ int dge_compact(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
     return DGE_OK;
 }
 
-int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
-              void *stream_)
+}  // extern "C"
+
+namespace {
+
+// dge_evict and dge_evict_inplace: validation, scores, selection, then the gather into the
+// packed outputs or into the cache itself.
+int evict_impl(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+               void *stream_, bool inplace)
 {
     Plan plan;
     int rc = make_plan(p, plan);
     if (rc != DGE_OK)
         return rc;
-    if (!bufs || !bufs->idx || !bufs->Kc || !bufs->Vc)
+    if (!bufs || !bufs->idx || (!inplace && (!bufs->Kc || !bufs->Vc)))
         return DGE_ERR_INVALID_ARG;
     if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK)
         return rc;
-    if (((uintptr_t)bufs->Kc & 15) || ((uintptr_t)bufs->Vc & 15) || ((uintptr_t)bufs->idx & 3) ||
-        ((uintptr_t)bufs->scores & 3) || !lse_ptrs_ok(bufs))
+    if ((!inplace && (((uintptr_t)bufs->Kc & 15) || ((uintptr_t)bufs->Vc & 15))) ||
+        ((uintptr_t)bufs->idx & 3) || ((uintptr_t)bufs->scores & 3) || !lse_ptrs_ok(bufs))
         return DGE_ERR_UNSUPPORTED;
     const Geometry &g = plan.g;
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    const TensorDesc K = desc(bufs->K), V = desc(bufs->V);
+    uint32_t *status = static_cast<uint32_t *>(ws);
     if (g.variant == DGE_VARIANT_STREAMING) {
         if (ws && ((uintptr_t)ws & 255))
             return DGE_ERR_UNSUPPORTED;
         if (ws)
             DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
-        DGE_LAUNCH("compact", stream, launch_compact(g, plan.layers, nullptr, bufs->idx, desc(bufs->K),
-                                      desc(bufs->V), bufs->Kc, bufs->Vc, true,
-                                      static_cast<uint32_t *>(ws), stream));
+        if (inplace)
+            DGE_LAUNCH("compact_inplace", stream,
+                       launch_compact_inplace(g, plan.layers, nullptr, bufs->idx, K, V, true,
+                                              status, stream));
+        else
+            DGE_LAUNCH("compact", stream,
+                       launch_compact(g, plan.layers, nullptr, bufs->idx, K, V, bufs->Kc,
+                                      bufs->Vc, true, status, stream));
         return DGE_OK;
     }
     if ((rc = check_tensor(bufs->Q)) != DGE_OK || (rc = check_ws(plan, ws, ws_bytes)) != DGE_OK)
         return rc;
     DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
-    const TensorDesc K = desc(bufs->K), V = desc(bufs->V), Q = desc(bufs->Q);
+    const TensorDesc Q = desc(bufs->Q);
     if ((rc = run_scoring(plan, K, Q, ws, stream, bufs->lse_in, bufs->lse_out)) != DGE_OK)
         return rc;
     float *raw = ws_at<float>(ws, plan.off_raw);
@@ -523,8 +536,50 @@ int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
     }
     if (!pool_select_supported(g))
         DGE_LAUNCH("select", stream, launch_select(g, plan.layers, sel, bufs->idx, stream));
-    DGE_LAUNCH("compact", stream, launch_compact(g, plan.layers, bufs->idx, nullptr, K, V, bufs->Kc, bufs->Vc,
-                                  false, static_cast<uint32_t *>(ws), stream));
+    if (inplace)
+        DGE_LAUNCH("compact_inplace", stream,
+                   launch_compact_inplace(g, plan.layers, bufs->idx, nullptr, K, V, false, status,
+                                          stream));
+    else
+        DGE_LAUNCH("compact", stream,
+                   launch_compact(g, plan.layers, bufs->idx, nullptr, K, V, bufs->Kc, bufs->Vc,
+                                  false, status, stream));
+    return DGE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+              void *stream)
+{
+    return evict_impl(p, bufs, ws, ws_bytes, stream, false);
+}
+
+int dge_evict_inplace(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws_bytes,
+                      void *stream)
+{
+    return evict_impl(p, bufs, ws, ws_bytes, stream, true);
+}
+
+int dge_compact_inplace(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
+                        const dge_tensor *V, void *ws, void *stream_)
+{
+    Plan plan;
+    int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    if (!idx || !K || !V)
+        return DGE_ERR_INVALID_ARG;
+    if ((rc = check_tensor(*K)) != DGE_OK || (rc = check_tensor(*V)) != DGE_OK)
+        return rc;
+    if (((uintptr_t)idx & 3) || ((uintptr_t)ws & 255))
+        return DGE_ERR_UNSUPPORTED;
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    DGE_LAUNCH("compact_inplace", stream,
+               launch_compact_inplace(plan.g, plan.layers, idx, nullptr, desc(*K), desc(*V),
+                                      false, static_cast<uint32_t *>(ws), stream));
     return DGE_OK;
 }
 

@@ -63,6 +63,12 @@ cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const flo
                           int32_t *idx, cudaStream_t stream);
 cudaError_t launch_streaming_indices(const Geometry &g, const LayerTable &layers, int32_t *idx,
                                      cudaStream_t stream);
+// In-place gather: rows [0, B_l) of every unit of K and V become the kept rows (idx ascending
+// per unit, as the selection writes it; implicit = StreamingLLM positions, written to idx_out).
+cudaError_t launch_compact_inplace(const Geometry &g, const LayerTable &layers,
+                                   const int32_t *idx_in, int32_t *idx_out, const TensorDesc &K,
+                                   const TensorDesc &V, bool implicit, uint32_t *status,
+                                   cudaStream_t stream);
 cudaError_t launch_compact(const Geometry &g, const LayerTable &layers, const int32_t *idx_in,
                            int32_t *idx_out, const TensorDesc &K, const TensorDesc &V, void *Kc,
                            void *Vc, bool implicit, uint32_t *status, cudaStream_t stream);

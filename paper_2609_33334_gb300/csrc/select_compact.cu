@@ -539,6 +539,84 @@ compact_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__ idx_out
     }
 }
 
+// In-place gather into the cache itself (Alg. 1: the cache of every head is edited once, in
+// place, temporal order kept): rows [0, B) of a unit become the kept rows.  Kept positions
+// ascend, so idx[r] >= r and a forward copy never overwrites a row still to be read.  One
+// CTA per unit walks its rows in chunks; inside a chunk every source row is read into
+// registers before the block barrier and written after it, so a row that is both read and
+// written within the chunk is read first; rows written by earlier chunks lie below every
+// later source row.  A position outside [r, n) is reported (DGE_ERR_INVALID_ARG) and skipped.
+template <int D>
+__global__ void __launch_bounds__(256)
+compact_inplace_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__ idx_out,
+                       TensorDesc K, TensorDesc V, SelectParams p, int implicit, uint32_t *status)
+{
+    constexpr int TPR = D / 8;             // threads per row (16 B each)
+    constexpr int RPI = 256 / TPR;          // rows per pass
+    constexpr int kPasses = 4;              // rows of a chunk: kPasses * RPI, in registers
+    const int64_t u = blockIdx.x;
+    int l, bb, h;
+    unit_coords(p.g, u, l, bb, h);
+    int budget;
+    const int64_t base = unit_row_base(p, u, budget);
+    __nv_bfloat16 *Ku = const_cast<__nv_bfloat16 *>(kv_unit_ptr(K, l, bb, h));
+    __nv_bfloat16 *Vu = const_cast<__nv_bfloat16 *>(kv_unit_ptr(V, l, bb, h));
+    const int part = threadIdx.x % TPR, rsub = threadIdx.x / TPR;
+    for (int r0 = 0; r0 < budget; r0 += kPasses * RPI) {
+        int4 kv[kPasses], vv[kPasses];
+        int dst[kPasses];
+#pragma unroll
+        for (int i = 0; i < kPasses; ++i) {
+            const int r = r0 + i * RPI + rsub;
+            dst[i] = -1;
+            if (r < budget) {
+                int pos;
+                if (implicit) {
+                    pos = r < p.g.sinks ? r : p.g.n - budget + r;
+                    if (part == 0 && idx_out)
+                        idx_out[base + r] = pos;
+                } else {
+                    pos = idx_in[base + r];
+                }
+                if (pos < r || pos >= p.g.n) {
+                    if (part == 0)
+                        set_status(status, DGE_ERR_INVALID_ARG);
+                } else if (pos != r) {
+                    kv[i] = *reinterpret_cast<const int4 *>(Ku + (int64_t)pos * K.s_pos + part * 8);
+                    vv[i] = *reinterpret_cast<const int4 *>(Vu + (int64_t)pos * V.s_pos + part * 8);
+                    dst[i] = r;
+                }
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int i = 0; i < kPasses; ++i)
+            if (dst[i] >= 0) {
+                *reinterpret_cast<int4 *>(Ku + (int64_t)dst[i] * K.s_pos + part * 8) = kv[i];
+                *reinterpret_cast<int4 *>(Vu + (int64_t)dst[i] * V.s_pos + part * 8) = vv[i];
+            }
+    }
+}
+
+cudaError_t launch_compact_inplace(const Geometry &g, const LayerTable &layers,
+                                   const int32_t *idx_in, int32_t *idx_out, const TensorDesc &K,
+                                   const TensorDesc &V, bool implicit, uint32_t *status,
+                                   cudaStream_t stream)
+{
+    SelectParams p;
+    p.g = g;
+    p.layers = layers;
+    if (g.U == 0)
+        return cudaSuccess;
+    if (g.d == 128)
+        compact_inplace_kernel<128><<<(unsigned)g.U, 256, 0, stream>>>(
+            idx_in, idx_out, K, V, p, implicit ? 1 : 0, status);
+    else
+        compact_inplace_kernel<64><<<(unsigned)g.U, 256, 0, stream>>>(
+            idx_in, idx_out, K, V, p, implicit ? 1 : 0, status);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_compact(const Geometry &g, const LayerTable &layers, const int32_t *idx_in,
                            int32_t *idx_out, const TensorDesc &K, const TensorDesc &V, void *Kc,
                            void *Vc, bool implicit, uint32_t *status, cudaStream_t stream)

@@ -159,3 +159,17 @@ def test_null_and_misaligned_arguments_rejected_before_launch(lib):
     assert lib.dge_compact(ctypes.byref(p), None, None, None, 0, 0, None, None) == \
         B.DGE_ERR_INVALID_ARG
     assert lib.dge_get_device_status(None, None) == B.DGE_ERR_INVALID_ARG
+    # in place: no Kc / Vc needed, idx still required and aligned
+    bufs.Kc = bufs.Vc = 0
+    assert lib.dge_evict(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value, None) == \
+        B.DGE_ERR_INVALID_ARG
+    bufs.idx = 0
+    assert lib.dge_evict_inplace(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value,
+                                 None) == B.DGE_ERR_INVALID_ARG
+    bufs.idx = 0x2002
+    assert lib.dge_evict_inplace(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value,
+                                 None) == B.DGE_ERR_UNSUPPORTED
+    assert lib.dge_compact_inplace(ctypes.byref(p), None, ctypes.byref(t), ctypes.byref(t), None,
+                                   None) == B.DGE_ERR_INVALID_ARG
+    assert lib.dge_compact_inplace(ctypes.byref(p), 0x2002, ctypes.byref(t), ctypes.byref(t),
+                                   None, None) == B.DGE_ERR_UNSUPPORTED
