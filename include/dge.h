@@ -223,6 +223,31 @@ int dge_evict_inplace(const dge_problem *p, const dge_buffers *bufs, void *ws, s
                       void *stream);
 
 /*
+ * Eviction diagnostics (Sec. "Attention-Mass Analysis"; Eq. evict-mass and Eq. match), SCORED
+ * only, for an eviction already done by dge_evict:
+ *   evicted_mass [L][b][Hq][m] (required): rho of every observation row, the share of its
+ *     softmax (over its visible keys) that falls on evicted keys: 1 - Z_hat / Z, where Z_hat
+ *     is the same sum over the retained keys only;
+ *   l_match [unit] (optional): the attention-matching loss of Eq. match, the mean over the
+ *     unit's rows of log Z - log Z_hat = -log(1 - rho);
+ *   run_length [unit] (optional): the mean contiguous run of retained positions,
+ *     B_l / (number of maximal runs of consecutive kept positions).
+ * Uses bufs->Q, bufs->Kc and bufs->idx as dge_evict wrote them, and bufs->lse_in = the rows'
+ * full-cache normalisers (dge_evict's lse_out, or the caller's own); K and V are not read.
+ * log Z_hat comes from the scoring run on each layer's packed kept keys as a cache of length
+ * B_l (the observation rows keep their relative positions), so the observation rows must lie
+ * in the protected tail (m <= tail; otherwise DGE_ERR_UNSUPPORTED).  ws: dge_workspace_size(p)
+ * bytes.
+ */
+typedef struct dge_diag {
+    float *evicted_mass;
+    float *l_match;
+    float *run_length;
+} dge_diag;
+int dge_diagnostics(const dge_problem *p, const dge_buffers *bufs, const dge_diag *out,
+                    void *ws, size_t ws_bytes, void *stream);
+
+/*
  * PyramidKV's per-layer past budgets (App. L): c = B - w, min = floor(c/20),
  * max = 2c - min, steps = floor((max - min)/(L - 1)), out[l] = max - l*steps.
  * These are past tokens only; add the protected tail to get dge budgets.

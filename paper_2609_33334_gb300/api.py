@@ -217,6 +217,25 @@ def evict_inplace(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torc
     return o
 
 
+def diagnostics(p: Problem, Q: torch.Tensor, evicted: dict, lse: torch.Tensor, *, ws=None,
+                stream=None) -> dict:
+    """dge_diagnostics: per-row evicted mass (Problem.lse_shape), and per unit the
+    attention-matching loss and the mean run of retained positions, for an eviction whose
+    outputs (``evicted["Kc"]``, ``evicted["idx"]``) came from evict(); ``lse`` = the rows'
+    full-cache normalisers (evict(..., want_lse=True)["lse"])."""
+    dev = Q.device
+    rho = torch.empty(p.lse_shape, dtype=torch.float32, device=dev)
+    lm = torch.empty(p.U, dtype=torch.float32, device=dev)
+    rl = torch.empty(p.U, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(p, dev)
+    bufs = B.dge_buffers(Q=B.tensor_desc(Q), Kc=B.ptr(evicted["Kc"]), idx=B.ptr(evicted["idx"]),
+                         lse_in=_lse_arg(p, lse))
+    out = B.dge_diag(evicted_mass=rho.data_ptr(), l_match=lm.data_ptr(), run_length=rl.data_ptr())
+    B.dge_diagnostics(p.c(), bufs, out, ws.data_ptr(), ws.numel(), _stream(stream))
+    return {"evicted_mass": rho, "l_match": lm, "run_length": rl}
+
+
 def device_status(ws: torch.Tensor, stream=None) -> int:
     """dge_get_device_status: sync the stream and read/clear the status word."""
     return B.dge_get_device_status(ws.data_ptr(), _stream(stream))

@@ -44,6 +44,10 @@ class dge_buffers(ctypes.Structure):
                 ("lse_out", c_void_p)]
 
 
+class dge_diag(ctypes.Structure):
+    _fields_ = [("evicted_mass", c_void_p), ("l_match", c_void_p), ("run_length", c_void_p)]
+
+
 class dge_kernel_time(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char * 48), ("launches", c_int64), ("total_ms", ctypes.c_double)]
 
@@ -72,6 +76,7 @@ _SIGS = {
     "dge_compact": [_P, c_void_p, _T, _T, c_void_p, c_void_p, c_void_p, c_void_p],
     "dge_evict": [_P, _B, c_void_p, c_size_t, c_void_p],
     "dge_evict_inplace": [_P, _B, c_void_p, c_size_t, c_void_p],
+    "dge_diagnostics": [_P, _B, ctypes.POINTER(dge_diag), c_void_p, c_size_t, c_void_p],
     "dge_compact_inplace": [_P, c_void_p, _T, _T, c_void_p, c_void_p],
     "dge_pyramid_budgets": [c_int32, c_int32, c_int32, POINTER(c_int32)],
     "dge_get_device_status": [c_void_p, c_void_p],
@@ -143,6 +148,12 @@ def dge_compact(p: dge_problem, idx: int, K: dge_tensor, V: dge_tensor, Kc: int,
                 ws: int, stream: int) -> None:
     _check("dge_compact", _lib().dge_compact(ctypes.byref(p), idx, ctypes.byref(K),
                                              ctypes.byref(V), Kc, Vc, ws, stream))
+
+
+def dge_diagnostics(p: dge_problem, bufs: dge_buffers, out: dge_diag, ws: int, ws_bytes: int,
+                    stream: int) -> None:
+    _check("dge_diagnostics", _lib().dge_diagnostics(ctypes.byref(p), ctypes.byref(bufs),
+                                                     ctypes.byref(out), ws, ws_bytes, stream))
 
 
 def dge_evict_inplace(p: dge_problem, bufs: dge_buffers, ws: int, ws_bytes: int,

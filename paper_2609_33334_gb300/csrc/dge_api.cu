@@ -563,6 +563,65 @@ int dge_evict_inplace(const dge_problem *p, const dge_buffers *bufs, void *ws, s
     return evict_impl(p, bufs, ws, ws_bytes, stream, true);
 }
 
+int dge_diagnostics(const dge_problem *p, const dge_buffers *bufs, const dge_diag *out,
+                    void *ws, size_t ws_bytes, void *stream_)
+{
+    Plan plan;
+    int rc = make_plan(p, plan);
+    if (rc != DGE_OK)
+        return rc;
+    const Geometry &g = plan.g;
+    if (g.variant != DGE_VARIANT_SCORED || !bufs || !out || !out->evicted_mass || !bufs->Kc ||
+        !bufs->idx || !bufs->lse_in)
+        return DGE_ERR_INVALID_ARG;
+    // The observation rows must lie in the protected tail, so that they are the last m rows of
+    // every layer's kept cache.
+    if (g.m > g.tail)
+        return DGE_ERR_UNSUPPORTED;
+    if ((rc = check_tensor(bufs->Q)) != DGE_OK || (rc = check_ws(plan, ws, ws_bytes)) != DGE_OK)
+        return rc;
+    if (((uintptr_t)bufs->Kc & 15) || ((uintptr_t)bufs->idx & 3) ||
+        ((uintptr_t)bufs->lse_in & 3) || ((uintptr_t)out->evicted_mass & 3) ||
+        ((uintptr_t)out->l_match & 3) || ((uintptr_t)out->run_length & 3))
+        return DGE_ERR_UNSUPPORTED;
+    // Each layer's kept keys as a cache of its own: n' = B_l rows, every one kept.
+    Plan sub[kMaxLayers];
+    for (int l = 0; l < g.L; ++l) {
+        dge_problem q = *p;
+        const int32_t B = plan.layers.budget[l];
+        q.num_layers = 1;
+        q.seq_len = B;
+        q.budgets = &plan.layers.budget[l];
+        q.pool = DGE_POOL_NONE;
+        q.pool_kernel = 1;
+        if ((rc = make_plan(&q, sub[l])) != DGE_OK)
+            return rc;
+        if (sub[l].ws_bytes > ws_bytes)
+            return DGE_ERR_WORKSPACE_TOO_SMALL;
+    }
+    cudaStream_t stream = static_cast<cudaStream_t>(stream_);
+    DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
+    const int64_t rows_per_layer = (int64_t)g.b * g.Hkv * g.R;  // lse entries of one layer
+    for (int l = 0; l < g.L; ++l) {
+        const int64_t B = plan.layers.budget[l];
+        dge_tensor kl;
+        kl.data = static_cast<const __nv_bfloat16 *>(bufs->Kc) + plan.layers.row_base[l] * g.d;
+        kl.stride_pos = g.d;
+        kl.stride_head = B * g.d;
+        kl.stride_batch = (int64_t)g.Hkv * B * g.d;
+        kl.stride_layer = (int64_t)g.b * g.Hkv * B * g.d;
+        TensorDesc Ql = desc(bufs->Q);
+        Ql.data += (int64_t)l * bufs->Q.stride_layer;
+        if ((rc = run_scoring(sub[l], desc(kl), Ql, ws, stream, nullptr,
+                              out->evicted_mass + (int64_t)l * rows_per_layer)) != DGE_OK)
+            return rc;
+    }
+    DGE_LAUNCH("diagnostics", stream,
+               launch_diag(bufs->lse_in, out->evicted_mass, bufs->idx, g, plan.layers,
+                           out->l_match, out->run_length, stream));
+    return DGE_OK;
+}
+
 int dge_compact_inplace(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
                         const dge_tensor *V, void *ws, void *stream_)
 {

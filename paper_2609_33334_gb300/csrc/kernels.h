@@ -54,6 +54,12 @@ cudaError_t launch_lse_import(const float *lse_in, float *lse2, int64_t total, c
 cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const float *lse2,
                               const uint32_t *ready, int64_t U, int R, float *lse_out,
                               cudaStream_t stream);
+// Diagnostics of one eviction from lse (full cache) and lse_hat (kept keys), both [U][R]
+// natural log: rho_io holds lse_hat on entry and the evicted mass on return; l_match and
+// run_length [U] (nullable).
+cudaError_t launch_diag(const float *lse, float *rho_io, const int32_t *idx, const Geometry &g,
+                        const LayerTable &layers, float *l_match, float *run_length,
+                        cudaStream_t stream);
 // Pooling and selection in one kernel (the evict path), for P <= 32768 positions per unit.
 // pooled_out (nullable) receives the pooled scores.
 bool pool_select_supported(const Geometry &g);

@@ -209,6 +209,37 @@ def test_missed_mass_identity_on_gathered_cache(oracle_lib):
     assert err <= 2 * beta * rho + 1e-12
 
 
+def test_evicted_mass_from_kept_cache_normaliser(oracle_lib):
+    """Eq. match: rho_q = sum over evicted visible keys of the row's softmax weights.
+
+    The diagnostics compute it as 1 - exp(lse_hat - lse), with lse_hat the normaliser of the
+    kept keys taken as a cache of length B (the observation rows in the kept tail keep their
+    relative positions).  Pinned against the definition, summed by brute force (pure Python,
+    math.fsum) over the evicted keys each row sees.
+    """
+    from oracle import brute
+    rng = np.random.default_rng(12)
+    n, d, m, G, budget = 90, 8, 3, 2, 30
+    K = _bf16_bits(rng.normal(size=(n, d)))
+    Q = _bf16_bits(rng.normal(size=(G * m, d)))
+    pos = oracle.scored_positions(n, m, G)
+    scale = 1.0 / np.sqrt(d)
+    idx = oracle.select(rng.random(n - m), n, 0, m, budget)      # tail [n-m, n) kept
+    _, lse = oracle.scores(Q[None], K[None], pos, n - m, scale, want_lse=True)
+    _, lse_hat = oracle.scores(Q[None], oracle.gather(K, idx)[None],
+                               oracle.scored_positions(budget, m, G), budget - m, scale,
+                               want_lse=True)
+    rho = -np.expm1(lse_hat[0] - lse[0])
+    Kf = [[brute.bf16_to_float(x) for x in row] for row in K]
+    kept = set(idx.tolist())
+    for r in range(G * m):
+        q = [brute.bf16_to_float(x) for x in Q[r]]
+        a = brute.attention_row(q, Kf[:pos[r] + 1], scale)
+        want = math.fsum(a[j] for j in range(pos[r] + 1) if j not in kept)
+        assert rho[r] == pytest.approx(want, rel=1e-9, abs=1e-13)
+    assert np.all((rho > 0) & (rho < 1))
+
+
 def _span_kept_counts(wl):
     t = inputs.make_inputs(wl)
     Q, K, V = (inputs.bf16_bits(t[x]) for x in "QKV")
