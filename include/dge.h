@@ -233,7 +233,8 @@ int dge_evict_inplace(const dge_problem *p, const dge_buffers *bufs, void *ws, s
  *   run_length [unit] (optional): the mean contiguous run of retained positions,
  *     B_l / (number of maximal runs of consecutive kept positions).
  * Uses bufs->Q, bufs->Kc and bufs->idx as dge_evict wrote them, and bufs->lse_in = the rows'
- * full-cache normalisers (dge_evict's lse_out, or the caller's own); K and V are not read.
+ * full-cache normalisers (dge_evict's lse_out, or the caller's own); bufs->K and bufs->V only
+ * for the held-out queries below.
  * log Z_hat comes from the scoring run on each layer's packed kept keys as a cache of length
  * B_l (the observation rows keep their relative positions), so the observation rows must lie
  * in the protected tail (m <= tail; otherwise DGE_ERR_UNSUPPORTED).  ws: dge_workspace_size(p)
@@ -243,6 +244,19 @@ typedef struct dge_diag {
     float *evicted_mass;
     float *l_match;
     float *run_length;
+    /* Optional held-out decode queries (heldout_q.data NULL: skipped): bf16 [L][b][Hq][d]
+     * through the tensor's strides (stride_pos unused), one query per head at position n, so
+     * it attends over all n keys of bufs->K / bufs->V (the cache before compaction).  With
+     * weights a_j = softmax_j(scale q.k_j), kept set R = the head's idx and evicted set E:
+     *   heldout_mass [L][b][Hq]: m(E) = sum_{j in E} a_j,
+     *   heldout_err  [L][b][Hq]: |o - o~|, o = sum_j a_j v_j, o~ = sum_{j in R} a_j v_j/(1-m),
+     *   heldout_gap  [L][b][Hq]: m(E) |mu_E - mu_R| with mu the a-weighted value means over
+     *     E and R; Eq. evict-mass says heldout_err equals it exactly.
+     * The three outputs are required when heldout_q.data is set. */
+    dge_tensor heldout_q;
+    float *heldout_mass;
+    float *heldout_err;
+    float *heldout_gap;
 } dge_diag;
 int dge_diagnostics(const dge_problem *p, const dge_buffers *bufs, const dge_diag *out,
                     void *ws, size_t ws_bytes, void *stream);

@@ -218,11 +218,14 @@ def evict_inplace(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torc
 
 
 def diagnostics(p: Problem, Q: torch.Tensor, evicted: dict, lse: torch.Tensor, *, ws=None,
-                stream=None) -> dict:
+                heldout_q: Optional[torch.Tensor] = None, K: Optional[torch.Tensor] = None,
+                V: Optional[torch.Tensor] = None, stream=None) -> dict:
     """dge_diagnostics: per-row evicted mass (Problem.lse_shape), and per unit the
     attention-matching loss and the mean run of retained positions, for an eviction whose
     outputs (``evicted["Kc"]``, ``evicted["idx"]``) came from evict(); ``lse`` = the rows'
-    full-cache normalisers (evict(..., want_lse=True)["lse"])."""
+    full-cache normalisers (evict(..., want_lse=True)["lse"]).  With ``heldout_q`` (bf16
+    [L][b][Hq][d]) and the full cache K, V: per query head the held-out evicted mass,
+    |o - o~| and m |mu_E - mu_R| (Eq. evict-mass)."""
     dev = Q.device
     rho = torch.empty(p.lse_shape, dtype=torch.float32, device=dev)
     lm = torch.empty(p.U, dtype=torch.float32, device=dev)
@@ -232,8 +235,24 @@ def diagnostics(p: Problem, Q: torch.Tensor, evicted: dict, lse: torch.Tensor, *
     bufs = B.dge_buffers(Q=B.tensor_desc(Q), Kc=B.ptr(evicted["Kc"]), idx=B.ptr(evicted["idx"]),
                          lse_in=_lse_arg(p, lse))
     out = B.dge_diag(evicted_mass=rho.data_ptr(), l_match=lm.data_ptr(), run_length=rl.data_ptr())
+    res = {"evicted_mass": rho, "l_match": lm, "run_length": rl}
+    if heldout_q is not None:
+        if heldout_q.dtype != torch.bfloat16 or heldout_q.dim() != 4 or \
+                tuple(heldout_q.shape) != (p.L, p.b, p.Hq, p.d) or heldout_q.stride(3) != 1:
+            raise ValueError(f"heldout_q must be bf16 [{p.L}][{p.b}][{p.Hq}][{p.d}]")
+        _check_cache(K, "K")
+        _check_cache(V, "V")
+        hq = heldout_q.unsqueeze(3)                      # [L][b][Hq][1][d] for the descriptor
+        for k in ("heldout_mass", "heldout_err", "heldout_gap"):
+            res[k] = torch.empty((p.L, p.b, p.Hq), dtype=torch.float32, device=dev)
+        out.heldout_q = B.tensor_desc(hq)
+        out.heldout_mass = res["heldout_mass"].data_ptr()
+        out.heldout_err = res["heldout_err"].data_ptr()
+        out.heldout_gap = res["heldout_gap"].data_ptr()
+        bufs.K = B.tensor_desc(K)
+        bufs.V = B.tensor_desc(V)
     B.dge_diagnostics(p.c(), bufs, out, ws.data_ptr(), ws.numel(), _stream(stream))
-    return {"evicted_mass": rho, "l_match": lm, "run_length": rl}
+    return res
 
 
 def device_status(ws: torch.Tensor, stream=None) -> int:

@@ -45,7 +45,9 @@ class dge_buffers(ctypes.Structure):
 
 
 class dge_diag(ctypes.Structure):
-    _fields_ = [("evicted_mass", c_void_p), ("l_match", c_void_p), ("run_length", c_void_p)]
+    _fields_ = [("evicted_mass", c_void_p), ("l_match", c_void_p), ("run_length", c_void_p),
+                ("heldout_q", dge_tensor), ("heldout_mass", c_void_p), ("heldout_err", c_void_p),
+                ("heldout_gap", c_void_p)]
 
 
 class dge_kernel_time(ctypes.Structure):

@@ -584,6 +584,16 @@ int dge_diagnostics(const dge_problem *p, const dge_buffers *bufs, const dge_dia
         ((uintptr_t)bufs->lse_in & 3) || ((uintptr_t)out->evicted_mass & 3) ||
         ((uintptr_t)out->l_match & 3) || ((uintptr_t)out->run_length & 3))
         return DGE_ERR_UNSUPPORTED;
+    if (out->heldout_q.data) {
+        if (!out->heldout_mass || !out->heldout_err || !out->heldout_gap)
+            return DGE_ERR_INVALID_ARG;
+        if ((rc = check_tensor(out->heldout_q)) != DGE_OK ||
+            (rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK)
+            return rc;
+        if (((uintptr_t)out->heldout_mass & 3) || ((uintptr_t)out->heldout_err & 3) ||
+            ((uintptr_t)out->heldout_gap & 3) || !heldout_supported(g))
+            return DGE_ERR_UNSUPPORTED;
+    }
     // Each layer's kept keys as a cache of its own: n' = B_l rows, every one kept.
     Plan sub[kMaxLayers];
     for (int l = 0; l < g.L; ++l) {
@@ -619,6 +629,11 @@ int dge_diagnostics(const dge_problem *p, const dge_buffers *bufs, const dge_dia
     DGE_LAUNCH("diagnostics", stream,
                launch_diag(bufs->lse_in, out->evicted_mass, bufs->idx, g, plan.layers,
                            out->l_match, out->run_length, stream));
+    if (out->heldout_q.data)
+        DGE_LAUNCH("heldout", stream,
+                   launch_heldout(desc(out->heldout_q), desc(bufs->K), desc(bufs->V), bufs->idx,
+                                  g, plan.layers, out->heldout_mass, out->heldout_err,
+                                  out->heldout_gap, stream));
     return DGE_OK;
 }
 

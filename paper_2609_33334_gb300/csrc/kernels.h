@@ -60,6 +60,12 @@ cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const floa
 cudaError_t launch_diag(const float *lse, float *rho_io, const int32_t *idx, const Geometry &g,
                         const LayerTable &layers, float *l_match, float *run_length,
                         cudaStream_t stream);
+// Held-out decode queries (one per query head, position n) against a kept set: evicted mass,
+// |o - o~| and m |mu_E - mu_R| per head (Eq. evict-mass).  n <= 131072.
+bool heldout_supported(const Geometry &g);
+cudaError_t launch_heldout(const TensorDesc &Qh, const TensorDesc &K, const TensorDesc &V,
+                           const int32_t *idx, const Geometry &g, const LayerTable &layers,
+                           float *mass, float *err, float *gap, cudaStream_t stream);
 // Pooling and selection in one kernel (the evict path), for P <= 32768 positions per unit.
 // pooled_out (nullable) receives the pooled scores.
 bool pool_select_supported(const Geometry &g);

@@ -76,3 +76,38 @@ def test_diagnostics_need_observation_rows_in_the_tail():
     with pytest.raises(B.DgeError) as e:
         api.diagnostics(p, tens["Q"], out, out["lse"])
     assert "UNSUPPORTED" in str(e.value).upper() or f"-> {B.DGE_ERR_UNSUPPORTED}" in str(e.value)
+
+
+@pytest.mark.parametrize("name", ["c1_tiny", "c3_small"])
+def test_heldout_query_evicted_mass_identity(name):
+    """Eq. evict-mass on held-out decode queries: |o - o~| = m(E) |mu_E - mu_R|, and each of
+    m(E), |o - o~| against a float64 evaluation of the definitions."""
+    wl = CASES[name]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    out = api.evict(p, tens["K"], tens["V"], tens["Q"], want_lse=True)
+    g = torch.Generator(device="cuda").manual_seed(7)
+    hq = torch.randn((wl.L, wl.b, wl.Hq, wl.d), generator=g, device="cuda").to(torch.bfloat16)
+    diag = api.diagnostics(p, tens["Q"], out, out["lse"], heldout_q=hq, K=tens["K"],
+                           V=tens["V"])
+    torch.cuda.synchronize()
+    mass, err, gap = (diag[k].double().cpu().numpy() for k in
+                      ("heldout_mass", "heldout_err", "heldout_gap"))
+    np.testing.assert_allclose(err, gap, rtol=2e-3, atol=1e-5)
+    scale = 1.0 / np.sqrt(wl.d)
+    Hf = hq.double().cpu().numpy()
+    for (l, b, hq_i) in [(0, 0, 0), (wl.L - 1, wl.b - 1, wl.Hq - 1), (0, wl.b - 1, wl.G)]:
+        h = hq_i // wl.G
+        r0, r1 = unit_rows(wl, l, b, h)
+        keep = np.zeros(wl.n, bool)
+        keep[out["idx"][r0:r1].cpu().numpy()] = True
+        Kf = tens["K"][l, b, h].double().cpu().numpy()
+        Vf = tens["V"][l, b, h].double().cpu().numpy()
+        s = Kf @ Hf[l, b, hq_i] * scale
+        a = np.exp(s - s.max())
+        a /= a.sum()
+        m = a[~keep].sum()
+        o = a @ Vf
+        mu_r = (a[keep] @ Vf[keep]) / (1 - m)
+        assert mass[l, b, hq_i] == pytest.approx(m, rel=1e-4, abs=1e-7)
+        assert err[l, b, hq_i] == pytest.approx(np.linalg.norm(o - mu_r), rel=2e-3, abs=1e-5)
