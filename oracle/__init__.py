@@ -74,6 +74,9 @@ def _load():
             lib.dgeo_pool.argtypes = [_f64p, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _f64p]
             lib.dgeo_select.argtypes = [_f64p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
                                         ctypes.c_int64, _i32p]
+            lib.dgeo_select_blocks.argtypes = [_f64p, ctypes.c_int64, ctypes.c_int64,
+                                               ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                               _i32p]
             lib.dgeo_streaming_indices.argtypes = [ctypes.c_int64, ctypes.c_int64,
                                                    ctypes.c_int64, _i32p]
             lib.dgeo_gather.argtypes = [_u8p, ctypes.c_int64, _i32p, ctypes.c_int64, _u8p]
@@ -156,6 +159,20 @@ def select(scores_by_pos: np.ndarray, n: int, s0: int, tail: int, budget: int) -
     return idx
 
 
+def select_blocks(scores_by_pos: np.ndarray, n: int, s0: int, tail: int, budget: int,
+                  bs: int) -> np.ndarray:
+    """Block-granular kept positions of one head, ascending (the "fixed b-blocks" rung;
+    the rule as read in dge_oracle.c): whole blocks of ``bs`` candidates by block-score sum,
+    the first block that does not fit contributing its lowest positions."""
+    P = n - tail
+    keep = budget - s0 - tail
+    s = np.ascontiguousarray(scores_by_pos[:P], dtype=np.float64)
+    idx = np.empty(budget, dtype=np.int32)
+    if _load().dgeo_select_blocks(_ptr(s, _f64p), P, n, s0, keep, bs, _ptr(idx, _i32p)) != 0:
+        raise ValueError("bad selection arguments")
+    return idx
+
+
 def streaming_indices(n: int, sinks: int, budget: int) -> np.ndarray:
     """StreamingLLM kept positions: [0, sinks) then the last budget - sinks (App. L)."""
     idx = np.empty(budget, dtype=np.int32)
@@ -187,6 +204,7 @@ def pyramid_budgets(B: int, w: int, L: int) -> np.ndarray:
 
 def evict_unit(Qg: np.ndarray, K: np.ndarray, V: np.ndarray, *, variant: int, m: int,
                tail: int, sinks: int, budget: int, pool_kind: int, kernel: int,
+               select_block: int = 0,
                scale: float | None = None) -> dict:
     """The whole pass for one KV head: scores -> pool -> select -> gather.
 
@@ -204,6 +222,7 @@ def evict_unit(Qg: np.ndarray, K: np.ndarray, V: np.ndarray, *, variant: int, m:
     P = n - tail
     raw = scores(Qg.reshape(1, G * rows, d), K[None], pos, P, scale)[0]
     pooled = pool(raw, pool_kind, kernel) if variant == 0 else raw.copy()
-    idx = select(pooled, n, sinks, tail, budget)
+    idx = select_blocks(pooled, n, sinks, tail, budget, select_block) if select_block > 1 \
+        else select(pooled, n, sinks, tail, budget)
     return {"raw": raw, "pooled": pooled, "idx": idx, "Kc": gather(K, idx),
             "Vc": gather(V, idx)}

@@ -208,6 +208,63 @@ int dgeo_select(const double *scores, int64_t P, int64_t n, int64_t s0, int64_t 
 }
 
 /*
+ * Block-granular retention: the selection ladder's "fixed b-blocks" rung (Table "Selection
+ * decomposition"; block sizes 8/16/32 in App. "Diagnostic details").  The paper names the rung
+ * but not its rule; this is the reading implemented here.  Candidates [s0, P) form consecutive
+ * blocks of bs positions starting at s0 (the last one may be shorter); a block's score is the
+ * sum of its positions' scores; blocks are taken whole in the order (score desc, block index
+ * asc) while they fit in `keep`, and the first block that does not fit gives its lowest
+ * keep - taken positions.  Output as dgeo_select.  bs = 1 is dgeo_select.
+ * Returns 0, or -1 on bad sizes / allocation failure.
+ */
+int dgeo_select_blocks(const double *scores, int64_t P, int64_t n, int64_t s0, int64_t keep,
+                       int64_t bs, int32_t *idx)
+{
+    if (s0 < 0 || s0 > P || P > n || keep < 0 || keep > P - s0 || bs < 1)
+        return -1;
+    const int64_t nc = P - s0, nb = (nc + bs - 1) / bs;
+    cand_t *blk = (cand_t *)malloc(sizeof(cand_t) * (size_t)(nb > 0 ? nb : 1));
+    int64_t *take = (int64_t *)calloc((size_t)(nb > 0 ? nb : 1), sizeof(int64_t));
+    if (!blk || !take) {
+        free(blk);
+        free(take);
+        return -1;
+    }
+    for (int64_t k = 0; k < nb; ++k) {
+        const int64_t lo = s0 + k * bs, hi = lo + bs < P ? lo + bs : P;
+        double sum = 0.0;
+        for (int64_t j = lo; j < hi; ++j)
+            sum += scores[j];
+        blk[k].score = sum;
+        blk[k].pos = k;   /* block index: cand_order's tie rule puts the lower block first */
+    }
+    qsort(blk, (size_t)nb, sizeof(cand_t), cand_order);
+    int64_t left = keep;
+    for (int64_t i = 0; i < nb && left > 0; ++i) {
+        const int64_t k = blk[i].pos, lo = s0 + k * bs;
+        const int64_t size = (lo + bs < P ? lo + bs : P) - lo;
+        if (size <= left) {
+            take[k] = size;
+            left -= size;
+        } else {
+            take[k] = left;
+            left = 0;
+        }
+    }
+    int64_t o = 0;
+    for (int64_t j = 0; j < s0; ++j)
+        idx[o++] = (int32_t)j;
+    for (int64_t k = 0; k < nb; ++k)
+        for (int64_t q = 0; q < take[k]; ++q)
+            idx[o++] = (int32_t)(s0 + k * bs + q);
+    for (int64_t j = P; j < n; ++j)
+        idx[o++] = (int32_t)j;
+    free(blk);
+    free(take);
+    return 0;
+}
+
+/*
  * StreamingLLM retention (App. L): [0, sinks) followed by the last
  * budget - sinks positions.  Returns 0, or -1 on bad sizes.
  */

@@ -240,6 +240,65 @@ def test_evicted_mass_from_kept_cache_normaliser(oracle_lib):
     assert np.all((rho > 0) & (rho < 1))
 
 
+def _blocks_brute(scores, n, s0, tail, budget, bs):
+    """The block rule written out plainly: rank blocks by (sum desc, index asc) with a Python
+    sort, take whole blocks while they fit, then a prefix of the first that does not."""
+    P = n - tail
+    keep = budget - s0 - tail
+    blocks = []
+    for k, lo in enumerate(range(s0, P, bs)):
+        pos = list(range(lo, min(lo + bs, P)))
+        total = 0.0                  # left to right, as the rule adds (not Python's sum())
+        for j in pos:
+            total += scores[j]
+        blocks.append((-total, k, pos))
+    blocks.sort(key=lambda t: (t[0], t[1]))
+    kept, left = [], keep
+    for _, _, pos in blocks:
+        if left == 0:
+            break
+        take = pos if len(pos) <= left else pos[:left]
+        kept += take
+        left -= len(take)
+    return sorted(range(s0)) + sorted(kept) + list(range(P, n))
+
+
+def test_block_selection(oracle_lib):
+    """The block-granular rule: bs = 1 is token selection exactly; a hand-worked case; a plain
+    Python version of the rule on random scores with ties; whole blocks plus at most one
+    prefix, exactly `budget` positions, ascending."""
+    rng = np.random.default_rng(13)
+    for trial in range(20):
+        n, s0, tail = int(rng.integers(20, 300)), int(rng.integers(0, 5)), int(rng.integers(1, 12))
+        P = n - tail
+        budget = int(rng.integers(s0 + tail, n + 1))
+        sc = rng.random(P).round(1)                  # many ties
+        np.testing.assert_array_equal(oracle.select_blocks(sc, n, s0, tail, budget, 1),
+                                      oracle.select(sc, n, s0, tail, budget))
+        for bs in (2, 8, 16, 32):
+            got = oracle.select_blocks(sc, n, s0, tail, budget, bs)
+            assert got.tolist() == _blocks_brute(sc.tolist(), n, s0, tail, budget, bs)
+            assert len(got) == budget and np.all(np.diff(got) > 0)
+            cand = [j for j in got.tolist() if s0 <= j < P]
+            blocks = {}
+            for j in cand:
+                blocks.setdefault((j - s0) // bs, []).append(j)
+            partial = [k for k, js in blocks.items()
+                       if len(js) < min(bs, P - (s0 + k * bs))]
+            assert len(partial) <= 1
+            for k in partial:                        # a prefix of its block
+                assert blocks[k] == list(range(s0 + k * bs, s0 + k * bs + len(blocks[k])))
+    # hand-worked: s0 = 1, tail = 2, n = 13 -> candidates [1, 11) in blocks of 4:
+    # [1..4] sum 1.0, [5..8] sum 2.0, [9, 10] sum 1.5; keep = 7 - 1 - 2 = 4 ... then budget 9
+    sc = np.array([9.0, .1, .2, .3, .4, .5, .5, .5, .5, 1.0, .5])
+    np.testing.assert_array_equal(oracle.select_blocks(sc, 13, 1, 2, 7, 4),
+                                  [0, 5, 6, 7, 8, 11, 12])          # block [5..8] whole
+    np.testing.assert_array_equal(oracle.select_blocks(sc, 13, 1, 2, 9, 4),
+                                  [0, 5, 6, 7, 8, 9, 10, 11, 12])   # then [9, 10] (fits)
+    np.testing.assert_array_equal(oracle.select_blocks(sc, 13, 1, 2, 10, 4),
+                                  [0, 1, 5, 6, 7, 8, 9, 10, 11, 12])  # then a prefix of [1..4]
+
+
 def _span_kept_counts(wl):
     t = inputs.make_inputs(wl)
     Q, K, V = (inputs.bf16_bits(t[x]) for x in "QKV")
