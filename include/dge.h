@@ -87,6 +87,15 @@ typedef struct dge_problem {
     int32_t pool;          /* DGE_POOL_* (SCORED only; H2O and STREAMING do not pool) */
     int32_t pool_kernel;   /* odd, 1..31, when pool != NONE */
     float scale;           /* logit scale; 0 means 1/sqrt(head_dim) */
+    int32_t select_block;  /* 0 (or 1): keep the best positions.  2..64: block-granular
+                              selection, the selection ladder's fixed-block rung (Table
+                              "Selection decomposition"; sizes 8/16/32 in App. "Diagnostic
+                              details"), read as: candidates [sinks, P) in consecutive blocks of
+                              this many positions from `sinks` (the last may be shorter), ranked
+                              by the sum of their scores (ties: lower block first), taken whole
+                              while they fit; the first block that does not fit gives its
+                              lowest positions, so the budget is met exactly.  At most 16384
+                              blocks per unit.  SCORED and H2O. */
     const int32_t *budgets;/* HOST array [L]: kept rows per unit of layer l, counting the
                               protected sinks and tail: sinks + tail <= budgets[l] <= n
                               (STREAMING: sinks <= budgets[l] <= n) */

@@ -31,12 +31,13 @@ class Problem:
     pool: int = B.DGE_POOL_NONE
     pool_kernel: int = 1
     scale: float = 0.0
+    select_block: int = 0
 
     def c(self) -> B.dge_problem:
         return B.make_problem(L=self.L, b=self.b, Hq=self.Hq, Hkv=self.Hkv, d=self.d, n=self.n,
                               m=self.m, tail=self.tail, sinks=self.sinks, variant=self.variant,
                               pool=self.pool, pool_kernel=self.pool_kernel, scale=self.scale,
-                              budgets=self.budgets)
+                              select_block=self.select_block, budgets=self.budgets)
 
     @property
     def U(self) -> int:

@@ -30,7 +30,7 @@ class dge_problem(ctypes.Structure):
                 ("num_kv_heads", c_int32), ("head_dim", c_int32), ("obs_rows", c_int32),
                 ("seq_len", c_int64), ("tail", c_int32), ("sinks", c_int32),
                 ("variant", c_int32), ("pool", c_int32), ("pool_kernel", c_int32),
-                ("scale", c_float), ("budgets", POINTER(c_int32))]
+                ("scale", c_float), ("select_block", c_int32), ("budgets", POINTER(c_int32))]
 
 
 class dge_tensor(ctypes.Structure):
@@ -218,12 +218,13 @@ def dge_trace_set(buffer: int, nbytes: int, cta: int = 0) -> None:
 # --- marshalling helpers --------------------------------------------------------------
 
 def make_problem(*, L, b, Hq, Hkv, d, n, m=0, tail=0, sinks=0, variant=DGE_VARIANT_SCORED,
-                 pool=DGE_POOL_NONE, pool_kernel=1, scale=0.0, budgets) -> dge_problem:
+                 pool=DGE_POOL_NONE, pool_kernel=1, scale=0.0, select_block=0,
+                 budgets) -> dge_problem:
     """A dge_problem; keeps the budgets array alive on the returned object."""
     arr = (c_int32 * len(budgets))(*[int(x) for x in budgets])
     p = dge_problem(num_layers=L, batch=b, num_q_heads=Hq, num_kv_heads=Hkv, head_dim=d,
                     obs_rows=m, seq_len=n, tail=tail, sinks=sinks, variant=variant, pool=pool,
-                    pool_kernel=pool_kernel, scale=scale,
+                    pool_kernel=pool_kernel, scale=scale, select_block=select_block,
                     budgets=ctypes.cast(arr, POINTER(c_int32)))
     p._budgets_keepalive = arr
     return p

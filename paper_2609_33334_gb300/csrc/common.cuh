@@ -11,6 +11,8 @@ namespace dge {
 
 constexpr int kMaxLayers = 256;
 constexpr int kMaxRows = 640;          // stacked observation rows per unit held on chip
+constexpr int kMaxSelectBlock = 64;     // largest block of block-granular selection
+constexpr int kMaxSelectBlocks = 16384; // blocks per unit it sorts in shared memory
 constexpr int kStatusBytes = 256;      // status region at the start of every workspace
 
 // Device status word values (same numbering as the ABI status codes).
@@ -38,6 +40,7 @@ struct Geometry {
     int tail, sinks;
     int variant;
     int pool, pool_kernel;
+    int select_block;  // 0: select positions; >= 2: select blocks of this many candidates
     float scale_log2;   // scale * log2(e): logits are kept in base-2 units
     int64_t U;          // units = L*b*Hkv
 };

@@ -193,6 +193,18 @@ int make_plan(const dge_problem *p, Plan &plan)
         }
     }
 
+    g.select_block = 0;
+    if (p->variant != DGE_VARIANT_STREAMING) {
+        if (p->select_block < 0 || p->select_block > kMaxSelectBlock)
+            return DGE_ERR_INVALID_ARG;
+        if (p->select_block >= 2) {
+            const int64_t C = (int64_t)g.P - g.sinks;
+            if ((C + p->select_block - 1) / p->select_block > kMaxSelectBlocks)
+                return DGE_ERR_UNSUPPORTED;
+            g.select_block = p->select_block;
+        }
+    }
+
     int64_t acc = 0;
     for (int l = 0; l < g.L; ++l) {
         const int32_t B = p->budgets[l];
@@ -451,7 +463,11 @@ int dge_select(const dge_problem *p, const float *scores, int32_t *idx, void *st
     }
     if (!scores || ((uintptr_t)scores & 3) != 0)
         return DGE_ERR_INVALID_ARG;
-    DGE_LAUNCH("select", stream, launch_select(plan.g, plan.layers, scores, idx, stream));
+    if (plan.g.select_block >= 2)
+        DGE_LAUNCH("block_select", stream,
+                   launch_block_select(plan.g, plan.layers, scores, idx, stream));
+    else
+        DGE_LAUNCH("select", stream, launch_select(plan.g, plan.layers, scores, idx, stream));
     return DGE_OK;
 }
 
@@ -522,7 +538,8 @@ int evict_impl(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t w
         return rc;
     float *raw = ws_at<float>(ws, plan.off_raw);
     const float *sel = raw;
-    if (pool_select_supported(g)) {
+    const bool fused = g.select_block < 2 && pool_select_supported(g);
+    if (fused) {
         DGE_LAUNCH("pool_select", stream,
                    launch_pool_select(g, plan.layers, raw, bufs->scores, bufs->idx, stream));
     } else if (g.pool != DGE_POOL_NONE) {
@@ -534,7 +551,10 @@ int evict_impl(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t w
                                        cudaMemcpyDeviceToDevice, stream),
                        "scores copy");
     }
-    if (!pool_select_supported(g))
+    if (g.select_block >= 2)
+        DGE_LAUNCH("block_select", stream,
+                   launch_block_select(g, plan.layers, sel, bufs->idx, stream));
+    else if (!fused)
         DGE_LAUNCH("select", stream, launch_select(g, plan.layers, sel, bufs->idx, stream));
     if (inplace)
         DGE_LAUNCH("compact_inplace", stream,

@@ -71,6 +71,9 @@ cudaError_t launch_heldout(const TensorDesc &Qh, const TensorDesc &K, const Tens
 bool pool_select_supported(const Geometry &g);
 cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, const float *raw,
                                float *pooled_out, int32_t *idx, cudaStream_t stream);
+// Block-granular selection (g.select_block >= 2) from final scores [U][P].
+cudaError_t launch_block_select(const Geometry &g, const LayerTable &layers, const float *scores,
+                                int32_t *idx, cudaStream_t stream);
 cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const float *scores,
                           int32_t *idx, cudaStream_t stream);
 cudaError_t launch_streaming_indices(const Geometry &g, const LayerTable &layers, int32_t *idx,

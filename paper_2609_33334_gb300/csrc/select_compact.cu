@@ -472,6 +472,126 @@ cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, cons
 }
 
 // ---------------------------------------------------------------------------
+// Block-granular selection (the selection ladder's fixed-block rung; the rule as read in
+// dge.h): one CTA per unit forms the block sums (fp32, positions in order), sorts the
+// (sum key, block index) pairs descending in shared memory (bitonic; pairs are unique, so the
+// order is deterministic), walks the ranking to take whole blocks while they fit and a prefix
+// of the first that does not, and writes the taken positions in block order (ascending).
+
+constexpr int kBsThreads = 1024;
+
+__global__ void __launch_bounds__(kBsThreads, 1)
+block_select_kernel(const float *__restrict__ scores, int32_t *__restrict__ idx, SelectParams p,
+                    int bs, int n2)
+{
+    extern __shared__ __align__(16) uint64_t items[];          // [n2]
+    int *take = reinterpret_cast<int *>(items + n2);           // [nb]
+    __shared__ int warp_tot[kSelWarps], warp_base[kSelWarps];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t u = blockIdx.x;
+    const Geometry &g = p.g;
+    int budget;
+    int32_t *out = idx + unit_row_base(p, u, budget);
+    const int P = g.P, s0 = g.sinks, tail = g.n - g.P;
+    const int C = P - s0;
+    const int keep = budget - s0 - tail;
+    for (int j = tid; j < s0; j += kBsThreads)
+        out[j] = j;
+    for (int j = tid; j < tail; j += kBsThreads)
+        out[s0 + keep + j] = P + j;
+    if (keep <= 0)
+        return;
+    if (keep >= C) {
+        for (int j = tid; j < C; j += kBsThreads)
+            out[s0 + j] = s0 + j;
+        return;
+    }
+    const int nb = (C + bs - 1) / bs;
+    const float *sc = scores + u * (int64_t)P + s0;
+    for (int k = tid; k < n2; k += kBsThreads) {
+        uint64_t item = 0;
+        if (k < nb) {
+            const int lo = k * bs, hi = min(lo + bs, C);
+            float sum = 0.f;
+            for (int j = lo; j < hi; ++j)
+                sum += sc[j];
+            item = ((uint64_t)float_key(sum) << 32) | (uint32_t)(0xFFFFFFFFu - (uint32_t)k);
+            take[k] = 0;
+        }
+        items[k] = item;
+    }
+    __syncthreads();
+    // Bitonic sort, descending: the largest sum first, then the lowest block index.
+    for (int size = 2; size <= n2; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int i = tid; i < (n2 >> 1); i += kBsThreads) {
+                const int pos = 2 * i - (i & (stride - 1));
+                const uint64_t a = items[pos], b = items[pos + stride];
+                const bool down = (pos & size) == 0;
+                if ((a < b) == down) {
+                    items[pos] = b;
+                    items[pos + stride] = a;
+                }
+            }
+            __syncthreads();
+        }
+    if (tid == 0) {
+        int left = keep;
+        for (int i = 0; i < nb && left > 0; ++i) {
+            const int k = (int)(0xFFFFFFFFu - (uint32_t)items[i]);
+            const int size = min(bs, C - k * bs);
+            const int t = size <= left ? size : left;
+            take[k] = t;
+            left -= t;
+        }
+    }
+    __syncthreads();
+    // Positions in block order: thread t owns blocks [t*per, (t+1)*per).
+    const int per = (nb + kBsThreads - 1) / kBsThreads;
+    const int k0 = min(nb, tid * per), k1 = min(nb, k0 + per);
+    int mine = 0;
+    for (int k = k0; k < k1; ++k)
+        mine += take[k];
+    int incl = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int o = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off)
+            incl += o;
+    }
+    if (lane == 31)
+        warp_tot[warp] = incl;
+    __syncthreads();
+    scan_warp_counts(warp_tot, warp_base);
+    __syncthreads();
+    int o = warp_base[warp] + incl - mine;
+    for (int k = k0; k < k1; ++k)
+        for (int q = 0; q < take[k]; ++q)
+            out[s0 + o++] = s0 + k * bs + q;
+}
+
+cudaError_t launch_block_select(const Geometry &g, const LayerTable &layers, const float *scores,
+                                int32_t *idx, cudaStream_t stream)
+{
+    SelectParams p;
+    p.g = g;
+    p.layers = layers;
+    const int C = g.P - g.sinks;
+    const int nb = max(1, (C + g.select_block - 1) / g.select_block);
+    int n2 = 1;
+    while (n2 < nb)
+        n2 <<= 1;
+    const size_t smem = (size_t)n2 * sizeof(uint64_t) + (size_t)nb * sizeof(int);
+    cudaError_t err = cudaFuncSetAttribute(block_select_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (err != cudaSuccess)
+        return err;
+    block_select_kernel<<<(unsigned)g.U, kBsThreads, smem, stream>>>(scores, idx, p,
+                                                                    g.select_block, n2);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // StreamingLLM indices: [0, sinks) then the last budget - sinks positions.
 __global__ void streaming_index_kernel(int32_t *__restrict__ idx, SelectParams p)
 {

@@ -43,10 +43,11 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_struct_layout_matches_c():
-    # int32 x6, int64, int32 x5, float, pointer
-    assert ctypes.sizeof(B.dge_problem) == 64
+    # int32 x6, int64, int32 x5, float, int32, pointer
+    assert ctypes.sizeof(B.dge_problem) == 72
     assert B.dge_problem.seq_len.offset == 24
-    assert B.dge_problem.budgets.offset == 56
+    assert B.dge_problem.select_block.offset == 56
+    assert B.dge_problem.budgets.offset == 64
     assert ctypes.sizeof(B.dge_tensor) == 40
     assert ctypes.sizeof(B.dge_buffers) == 3 * 40 + 6 * 8
     assert B.dge_buffers.lse_in.offset == 3 * 40 + 4 * 8
@@ -102,6 +103,9 @@ def _problem(**kw):
     (dict(tail=1025), B.DGE_ERR_INVALID_ARG),
     (dict(m=100, Hq=64, Hkv=8), B.DGE_ERR_UNSUPPORTED),      # R = 800 rows > on-chip limit
     (dict(variant=5), B.DGE_ERR_INVALID_ARG),
+    (dict(select_block=65), B.DGE_ERR_INVALID_ARG),
+    (dict(select_block=-1), B.DGE_ERR_INVALID_ARG),
+    (dict(n=100000, select_block=2, budgets=[128]), B.DGE_ERR_UNSUPPORTED),   # > 16384 blocks
     (dict(L=300, budgets=[128] * 300), B.DGE_ERR_INVALID_ARG),
 ])
 def test_problem_validation(lib, kw, code):
