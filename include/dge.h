@@ -324,7 +324,9 @@ int dge_profile_end(dge_kernel_time *out, int capacity, int *count);
  * the MMA warp sees it landed, 21 when its accumulator is free, 22 when its MMAs
  * are issued and committed, 23 when the first epilogue warp has the result.  `bytes`
  * must cover the slots;
- * pass NULL to stop.  Host-side state, per process.
+ * pass NULL to stop.  Host-side state, per process.  Only launches that take a
+ * unit's query rows whole are traced; a launch split into row blocks (more stacked
+ * rows than one accumulator holds) writes nothing.
  */
 #define DGE_TRACE_SLOTS 24
 #define DGE_TRACE_LEN 4096

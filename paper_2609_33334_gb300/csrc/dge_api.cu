@@ -121,7 +121,7 @@ struct Plan {
     int nchunks = 0;
     TcPlan tc = {};          // tensor-core path decomposition (SCORED only)
     size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, off_count = 0,
-           off_ready = 0, ws_bytes = 0;
+           off_ready = 0, off_rawfx = 0, off_unitflag = 0, ws_bytes = 0;
 };
 
 constexpr int kScoredChunkKeys = 2048;
@@ -230,9 +230,12 @@ int make_plan(const dge_problem *p, Plan &plan)
         plan.nchunks = (g.n + plan.chunk_keys - 1) / plan.chunk_keys;
         // The partial region serves both scoring paths (the larger of the two layouts).
         size_t part_bytes = (size_t)g.U * g.R * plan.nchunks * sizeof(float2);
+        int nrb = 1;
         if (p->variant == DGE_VARIANT_SCORED) {
             plan.tc = tc_plan(g);
-            const size_t tc_bytes = (size_t)g.U * plan.tc.r4 * plan.tc.nchunks * sizeof(float);
+            nrb = plan.tc.nrb;
+            const size_t tc_bytes =
+                (size_t)g.U * nrb * plan.tc.r4 * plan.tc.nchunks * sizeof(float);
             if (tc_bytes > part_bytes)
                 part_bytes = tc_bytes;
         }
@@ -246,9 +249,17 @@ int make_plan(const dge_problem *p, Plan &plan)
         if (g.pool != DGE_POOL_NONE)
             off = align256(off + (size_t)g.U * g.P * sizeof(float));
         plan.off_count = off;
-        off = align256(off + (size_t)g.U * sizeof(uint32_t));
+        off = align256(off + (size_t)g.U * nrb * sizeof(uint32_t));
         plan.off_ready = off;
-        off = align256(off + (size_t)g.U * sizeof(uint32_t));
+        off = align256(off + (size_t)g.U * nrb * sizeof(uint32_t));
+        if (nrb > 1) {
+            // Row blocks of one unit add their column sums in fixed point (exact, so the
+            // order of the additions does not matter), and their range flags per unit.
+            plan.off_rawfx = off;
+            off = align256(off + (size_t)g.U * g.P * sizeof(unsigned long long));
+            plan.off_unitflag = off;
+            off = align256(off + (size_t)g.U * sizeof(uint32_t));
+        }
     }
     plan.ws_bytes = off;
     return DGE_OK;
@@ -325,11 +336,22 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
             tb.ready = nullptr;
             tb.status = static_cast<uint32_t *>(ws);
             tb.lse_in = lse_in;
+            unsigned long long *raw_fx = nullptr;
+            if (plan.tc.nrb > 1) {
+                raw_fx = ws_at<unsigned long long>(ws, plan.off_rawfx);
+                DGE_CHECK_CUDA(cudaMemsetAsync(raw_fx, 0, (size_t)g.U * g.P * 8, stream),
+                               "sum clear");
+                tb.raw_fx = raw_fx;
+            }
             bool encoded = false;
             DGE_LAUNCH("score_tc_lse", stream,
                        launch_score_tc(K, Q, g, plan.tc, tb, stream, &encoded));
-            if (encoded)
+            if (encoded) {
+                if (raw_fx)
+                    DGE_LAUNCH("fixed_to_float", stream,
+                               launch_fixed_to_float(raw_fx, raw, g.U * g.P, stream));
                 return DGE_OK;
+            }
         }
         DGE_LAUNCH("lse_import", stream, launch_lse_import(lse_in, lse2, g.U * g.R, stream));
         if (g.variant == DGE_VARIANT_H2O)
@@ -342,10 +364,10 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
     if (g.variant == DGE_VARIANT_SCORED && want_tc(g)) {
         uint32_t *count = ws_at<uint32_t>(ws, plan.off_count);
         uint32_t *ready = ws_at<uint32_t>(ws, plan.off_ready);
-        DGE_CHECK_CUDA(cudaMemsetAsync(count, 0, (size_t)g.U * sizeof(uint32_t), stream),
+        const size_t nsub = (size_t)g.U * plan.tc.nrb;   // sub-units (row blocks)
+        DGE_CHECK_CUDA(cudaMemsetAsync(count, 0, nsub * sizeof(uint32_t), stream),
                        "counter clear");
-        DGE_CHECK_CUDA(cudaMemsetAsync(ready, 0, (size_t)g.U * sizeof(uint32_t), stream),
-                       "flag clear");
+        DGE_CHECK_CUDA(cudaMemsetAsync(ready, 0, nsub * sizeof(uint32_t), stream), "flag clear");
         TcBuffers tb;
         tb.part = reinterpret_cast<float *>(partial);
         tb.lse2 = lse2;
@@ -353,22 +375,38 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
         tb.count = count;
         tb.ready = ready;
         tb.status = static_cast<uint32_t *>(ws);
+        const int nrb = plan.tc.nrb;
+        unsigned long long *raw_fx = nullptr;
+        uint32_t *unit_flag = ready;      // per-unit range flags for the recompute
+        if (nrb > 1) {
+            raw_fx = ws_at<unsigned long long>(ws, plan.off_rawfx);
+            DGE_CHECK_CUDA(cudaMemsetAsync(raw_fx, 0, (size_t)g.U * g.P * 8, stream),
+                           "sum clear");
+            tb.raw_fx = raw_fx;
+            unit_flag = ws_at<uint32_t>(ws, plan.off_unitflag);
+        }
         bool encoded = false;
         DGE_LAUNCH("score_tc", stream,
                    launch_score_tc(K, Q, g, plan.tc, tb, stream, &encoded));
         if (encoded) {
-            // Units whose row sums left fp32's safe range (ready == 2) are recomputed
-            // with the running-maximum kernels; every other unit returns at once.
+            if (nrb > 1) {
+                DGE_LAUNCH("fixed_to_float", stream,
+                           launch_fixed_to_float(raw_fx, raw, g.U * g.P, stream));
+                DGE_LAUNCH("unit_flags", stream,
+                           launch_unit_flags(ready, nrb, g.U, unit_flag, stream));
+            }
+            // Units whose row sums left fp32's safe range (flag 2) are recomputed with the
+            // running-maximum kernels; every other unit returns at once.
             DGE_LAUNCH("recompute_lse", stream,
-                       launch_lse_partial(K, Q, g, g.R, g.n, partial, stream, ready));
+                       launch_lse_partial(K, Q, g, g.R, g.n, partial, stream, unit_flag));
             DGE_LAUNCH("recompute_combine", stream,
-                       launch_combine_lse(partial, g.U * g.R, 1, lse2, stream, ready, g.R));
+                       launch_combine_lse(partial, g.U * g.R, 1, lse2, stream, unit_flag, g.R));
             DGE_LAUNCH("recompute_colsum", stream,
-                       launch_colsum_rows(K, Q, g, g.P, lse2, raw, stream, ready));
+                       launch_colsum_rows(K, Q, g, g.P, lse2, raw, stream, unit_flag));
             if (lse_out)
                 DGE_LAUNCH("lse_export", stream,
-                           launch_lse_export(tb.part, plan.tc.nchunks, plan.tc.r4, lse2, ready,
-                                             g.U, g.R, lse_out, stream));
+                           launch_lse_export(tb.part, plan.tc.nchunks, plan.tc.r4, lse2,
+                                             unit_flag, g.U, g.R, plan.tc.rows, lse_out, stream));
             return DGE_OK;
         }
     }
@@ -381,7 +419,8 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
         DGE_LAUNCH("colsum_rows", stream, launch_colsum_rows(K, Q, g, kScoredChunkKeys, lse2, raw, stream));
     if (lse_out)
         DGE_LAUNCH("lse_export", stream,
-                   launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, lse_out, stream));
+                   launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
+                                     stream));
     return DGE_OK;
 }
 

@@ -21,15 +21,19 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
 // Scoring on the tcgen05 path (score_tc.cu).
 struct TcPlan {
     int r_pad, nslab, chunk_keys, nchunks, kstages;
-    int r4;            // row stride of the chunk sums: R rounded up to 4 (16-byte rows)
+    int r4;            // row stride of the chunk sums: rows rounded up to 4 (16-byte rows)
+    int gsub = 1;      // query heads per sub-unit (row block)
+    int nrb = 1;       // sub-units per unit: G / gsub
+    int rows = 0;      // stacked rows of a sub-unit: gsub * m
     size_t smem;
 };
 struct TcBuffers {
-    float *part;       // [U][nchunks][r4] row sums of each key chunk
+    float *part;       // [U*nrb][nchunks][r4] row sums of each key chunk
     float *lse2;       // [U][R]
     float *raw;        // [U][P]
-    uint32_t *count;   // [U], zero before the launch
-    uint32_t *ready;   // [U], zero before the launch; 2 = recompute
+    unsigned long long *raw_fx = nullptr;  // [U][P], nrb > 1: fixed-point sums (2^-40)
+    uint32_t *count;   // [U*nrb], zero before the launch
+    uint32_t *ready;   // [U*nrb], zero before the launch; 2 = recompute
     uint32_t *status;
     const float *lse_in = nullptr;  // [U][R] supplied natural-log normalisers (one pass)
 };
@@ -52,7 +56,13 @@ cudaError_t launch_pool(const float *raw, float *out, int64_t U, int P, int pool
 // path, its chunk sums part [U][nchunks][r4] for units with ready != 2) -> natural-log out.
 cudaError_t launch_lse_import(const float *lse_in, float *lse2, int64_t total, cudaStream_t stream);
 cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const float *lse2,
-                              const uint32_t *ready, int64_t U, int R, float *lse_out,
+                              const uint32_t *ready, int64_t U, int R, int rows, float *lse_out,
+                              cudaStream_t stream);
+// Fixed-point (2^-40) column sums of row blocks -> float; per-unit range flags from the
+// flags of its nrb row blocks.
+cudaError_t launch_fixed_to_float(const unsigned long long *fx, float *out, int64_t total,
+                                  cudaStream_t stream);
+cudaError_t launch_unit_flags(const uint32_t *sub_flag, int nrb, int64_t U, uint32_t *unit_flag,
                               cudaStream_t stream);
 // Diagnostics of one eviction from lse (full cache) and lse_hat (kept keys), both [U][R]
 // natural log: rho_io holds lse_hat on entry and the evicted mass on return; l_match and

@@ -23,11 +23,12 @@ __global__ void lse_import_kernel(const float *__restrict__ in, float *__restric
 }
 
 // out[u][r] = ln 2 * lse2 of the row: from the tensor-core path's chunk sums (added in chunk
-// order, as that kernel merges them) unless the unit was recomputed (ready == 2) or there are
-// no chunk sums (warp-level path), then from lse2.
+// order, as that kernel merges them; row r of unit u is row r % rows of sub-unit
+// u * (R / rows) + r / rows) unless the unit was recomputed (ready == 2) or there are no chunk
+// sums (warp-level path), then from lse2.
 __global__ void lse_export_kernel(const float *__restrict__ part, int nchunks, int r4,
                                   const float *__restrict__ lse2,
-                                  const uint32_t *__restrict__ ready, int64_t U, int R,
+                                  const uint32_t *__restrict__ ready, int64_t U, int R, int rows,
                                   float *__restrict__ out)
 {
     const int64_t total = U * (int64_t)R;
@@ -38,7 +39,8 @@ __global__ void lse_export_kernel(const float *__restrict__ part, int nchunks, i
         float l2;
         if (part && !(ready && ready[u] == 2)) {
             float Z = 0.f;
-            const float *pu = part + u * (int64_t)nchunks * r4 + r;
+            const int64_t sub = u * (R / rows) + r / rows;
+            const float *pu = part + sub * (int64_t)nchunks * r4 + r % rows;
             for (int c = 0; c < nchunks; ++c)
                 Z += pu[(int64_t)c * r4];
             l2 = log2f(Z);
@@ -46,6 +48,28 @@ __global__ void lse_export_kernel(const float *__restrict__ part, int nchunks, i
             l2 = lse2[i];
         }
         out[i] = l2 * 0.69314718055994531f;
+    }
+}
+
+// Column sums of row blocks, added in fixed point (2^-40 units), back to float.
+__global__ void fixed_to_float_kernel(const unsigned long long *__restrict__ fx,
+                                      float *__restrict__ out, int64_t total)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x)
+        out[i] = (float)((double)(long long)fx[i] * 0x1p-40);
+}
+
+// A unit is recomputed when any of its row blocks left fp32's range.
+__global__ void unit_flags_kernel(const uint32_t *__restrict__ sub_flag, int nrb, int64_t U,
+                                  uint32_t *__restrict__ unit_flag)
+{
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U;
+         u += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t f = 0;
+        for (int rb = 0; rb < nrb; ++rb)
+            f = max(f, sub_flag[u * nrb + rb]);
+        unit_flag[u] = f;
     }
 }
 
@@ -64,11 +88,25 @@ cudaError_t launch_lse_import(const float *lse_in, float *lse2, int64_t total, c
 }
 
 cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const float *lse2,
-                              const uint32_t *ready, int64_t U, int R, float *lse_out,
+                              const uint32_t *ready, int64_t U, int R, int rows, float *lse_out,
                               cudaStream_t stream)
 {
     lse_export_kernel<<<blocks_for(U * (int64_t)R), 256, 0, stream>>>(part, nchunks, r4, lse2,
-                                                                       ready, U, R, lse_out);
+                                                                       ready, U, R, rows, lse_out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fixed_to_float(const unsigned long long *fx, float *out, int64_t total,
+                                  cudaStream_t stream)
+{
+    fixed_to_float_kernel<<<blocks_for(total), 256, 0, stream>>>(fx, out, total);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_unit_flags(const uint32_t *sub_flag, int nrb, int64_t U, uint32_t *unit_flag,
+                              cudaStream_t stream)
+{
+    unit_flags_kernel<<<blocks_for(U), 256, 0, stream>>>(sub_flag, nrb, U, unit_flag);
     return cudaGetLastError();
 }
 

@@ -69,6 +69,8 @@ constexpr int kFlagAbort = 0, kFlagKArm = 4, kFlagQArm = 8, kFlagSArm = 10;
 
 struct TcArgs {
     Geometry g;
+    int rows;          // stacked rows of a sub-unit: gsub heads x m (all of R when nrb == 1)
+    int nrb, gsub;     // sub-units (row blocks) per unit, query heads per sub-unit
     int r_pad, r4, nslab, kstages;
     int acc_stride;    // TMEM columns between accumulator buffers
     int unit_tiles, nchunks;   // key tiles of a unit; chunk c = tiles [c*T/nc, (c+1)*T/nc)
@@ -81,7 +83,8 @@ struct TcArgs {
     int64_t steps;
     float *part;       // [U][nchunks][r4]
     float *lse2;       // [U][R]
-    float *raw;        // [U][P]
+    float *raw;        // [U][P] (nrb == 1)
+    unsigned long long *raw_fx;  // [U][P] fixed point, 2^-40 units (nrb > 1): row blocks add
     uint32_t *count;   // [U]
     uint32_t *ready;   // [U]
     uint32_t *status;
@@ -175,6 +178,7 @@ struct Smem {
     float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
     float *xch;          // [kAccBufs][kEpiWG][128] phase-2 partial column sums
+    int *xcnt;           // [kAccBufs][4] arrivals (row-block path: exactly one finaliser)
 };
 
 __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
@@ -185,7 +189,7 @@ __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
            + kStageBytes                          // lse merge staging
            + kCtrlBytes                           // barriers, tmem holder, flags
            + (2 * 256 + 2 * kEpiWG * 4 * kMaxGroups * 16) * 4 + 16
-           + kAccBufs * kEpiWG * kTile * 4;
+           + kAccBufs * kEpiWG * kTile * 4 + kAccBufs * 4 * 4;
 }
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
@@ -213,6 +217,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int ks
     s.sLbad = reinterpret_cast<int *>(raw + off);
     off += 16;
     s.xch = reinterpret_cast<float *>(raw + off);
+    off += kAccBufs * kEpiWG * kTile * 4;
+    s.xcnt = reinterpret_cast<int *>(raw + off);
     return s;
 }
 
@@ -369,8 +375,10 @@ __device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
 }
 
 // kTr: with the cycle accounting and timelines of dge_trace_set (a separate build, so the
-// clock reads cost nothing when tracing is off).
-template <bool kTr>
+// clock reads cost nothing when tracing is off).  kFx: units split into row blocks whose
+// column sums meet in fixed point (a separate build, so the whole-unit path carries none of
+// it: its epilogue is latency-bound and slowed by 5% with it).
+template <bool kTr, bool kFx>
 __global__ void __launch_bounds__(kThreads, 1)
 score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
                 const TcArgs a)
@@ -411,19 +419,21 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         flag[kFlagSArm] = -1;
         // Phase-2 exchange: one barrier per accumulator and lane quarter, one arrival per
         // warpgroup.
-        for (int i = 0; i < kAccBufs * 4; ++i)
+        for (int i = 0; i < kAccBufs * 4; ++i) {
             ptx::mbar_init(&sm.bar[kBarXch + i], kEpiWG);
+            sm.xcnt[i] = 0;
+        }
         ptx::fence_mbar_init();
     }
     // Query rows R .. r_pad-1 are never written by TMA: zero them once so the padded
     // accumulator columns are exactly 0.
     {
-        const int pad_rows = a.r_pad - g.R;
+        const int pad_rows = a.r_pad - a.rows;
         const int words = pad_rows * 128 / 16;
         for (int b = 0; b < 2; ++b)
             for (int s = 0; s < a.nslab; ++s) {
                 int4 *base = reinterpret_cast<int4 *>(sm.q + ((size_t)b * a.nslab + s) * q_slab_bytes +
-                                                      (size_t)g.R * 128);
+                                                      (size_t)a.rows * 128);
                 for (int i = threadIdx.x; i < words; i += blockDim.x)
                     base[i] = make_int4(0, 0, 0, 0);
             }
@@ -460,7 +470,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     if (!get_task(a, t, j, T))
                         continue;
                     int l, bb, h;
-                    unit_coords(g, T.u, l, bb, h);
+                    unit_coords(g, kFx ? T.u / a.nrb : T.u, l, bb, h);
+                    const int qhead = h * g.G + (kFx ? (int)(T.u % a.nrb) * a.gsub : 0);
                     long long c0 = tclock<kTr>();
                     if (!wait_bar(&sm.bar[kBarQEmpty + qb], qph ^ 1, flag, a)) {
                         ok = false;
@@ -468,11 +479,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     }
                     cy_wq += tclock<kTr>() - c0;
                     ptx::mbar_arrive_expect_tx(&sm.bar[kBarQFull + qb],
-                                               (uint32_t)a.nslab * 128u * (uint32_t)g.R);
+                                               (uint32_t)a.nslab * 128u * (uint32_t)a.rows);
                     flag[kFlagQArm + qb] = (int)qph;
                     for (int s = 0; s < a.nslab; ++s)
                         ptx::tma_load_5d_hint(sm.q + ((size_t)qb * a.nslab + s) * q_slab_bytes,
-                                              &tmQ, &sm.bar[kBarQFull + qb], s * 64, 0, h * g.G,
+                                              &tmQ, &sm.bar[kBarQFull + qb], s * 64, 0, qhead,
                                               bb, l, keep);
                     qb ^= 1;
                     if (qb == 0)
@@ -641,9 +652,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 if (a.lse_in) {
                     // Supplied normalisers: -lse in base 2, straight from the caller's array.
                     float *L = sm.sL + lb * 256;
-                    const float *src = a.lse_in + T.u * g.R;
+                    const float *src = a.lse_in + T.u * a.rows;
                     for (int r = lane; r < a.r_pad; r += 32)
-                        L[r] = (got && r < g.R) ? -__ldg(src + r) * 1.4426950408889634f
+                        L[r] = (got && r < a.rows) ? -__ldg(src + r) * 1.4426950408889634f
                                                 : -INFINITY;
                     __syncwarp();
                     if (lane == 0) {
@@ -686,7 +697,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
 #pragma unroll
                         for (int i = 0; i < kRowsPerLane; ++i) {
                             const int r = lane + 32 * i;
-                            if (r < g.R)
+                            if (r < a.rows)
                                 Z[i] += sm.stage[c * a.r4 + r];
                         }
                 }
@@ -697,7 +708,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     const int r = lane + 32 * i;
                     if (r < a.r_pad) {
                         float v = -INFINITY;
-                        if (got && r < g.R) {
+                        if (got && r < a.rows) {
                             if (!(Z[i] >= 0x1p-60f && Z[i] < 0x1p126f))
                                 bad = true;
                             v = -log2f(Z[i]);
@@ -728,7 +739,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 if (ok) {
                     constexpr int W = kMaxGroups * 16;
                     float *dst = a.part + (T.u * a.nchunks + T.chunk) * a.r4;
-                    for (int col = lane; col < g.R; col += 32) {
+                    for (int col = lane; col < a.rows; col += 32) {
                         int w = 0;
                         while (w + 1 < kEpiWG && col >= a.gbase[w + 1] * 16)
                             ++w;
@@ -912,6 +923,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     if (ew == 0 && lane == 0)
                         trace_at<kTr>(a, kTrTimeline, 2048 + 2 * (p2c - 1) + 1);
                     task_ok = task_ok && !dead;
+                    // This unit's score row: plain stores, or fixed-point adds when it is
+                    // split into row blocks.
+                    const int64_t row_at = (int64_t)(kFx ? T.u / a.nrb : T.u) * g.P;
+                    float *const raw_row = kFx ? nullptr : a.raw + row_at;
+                    unsigned long long *const fx_row = kFx ? a.raw_fx + row_at : nullptr;
                     cy_p2s += tclock<kTr>() - c_start;
                     for (int tile = 0; tile < T.ntiles; ++tile, ++tc) {
                         const int ab = tc % kAccBufs;
@@ -947,8 +963,18 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         // both find it so: they store the same value).
                         int last = 0;
                         if (lane == 0) {
-                            uint64_t *xb = &sm.bar[kBarXch + ab * 4 + quarter];
-                            last = ptx::mbar_test_token(xb, ptx::mbar_arrive_token(xb)) ? 1 : 0;
+                            if (kFx) {
+                                // Row blocks add their sums atomically, so exactly one warp may
+                                // finalise: the one whose count completes the three arrivals.
+                                __threadfence_block();
+                                last = atomicAdd(&sm.xcnt[ab * 4 + quarter], 1) % kEpiWG ==
+                                       kEpiWG - 1;
+                                __threadfence_block();
+                            } else {
+                                uint64_t *xb = &sm.bar[kBarXch + ab * 4 + quarter];
+                                last = ptx::mbar_test_token(xb, ptx::mbar_arrive_token(xb)) ? 1
+                                                                                           : 0;
+                            }
                         }
                         last = __shfl_sync(0xffffffffu, last, 0);
                         __syncwarp();  // lane 0's acquire orders the other lanes' reads
@@ -957,8 +983,16 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
 #pragma unroll
                             for (int w = 1; w < kEpiWG; ++w)
                                 total += xs[w * kTile + kl];
-                            if (task_ok && key < T.k_hi)
-                                a.raw[T.u * g.P + key] = total;
+                            if (task_ok && key < T.k_hi) {
+                                // Row blocks of one unit add up exactly in integers; the scaling
+                                // by 2^40 is exact in fp32, so this matches a rounding of the
+                                // exact product.
+                                if (kFx)
+                                    atomicAdd(fx_row + key,
+                                              (unsigned long long)__float2ll_rn(total * 0x1p40f));
+                                else
+                                    raw_row[key] = total;
+                            }
                         }
                         cy_xch += tclock<kTr>() - cx;
                         release_acc(ab, 1u);
@@ -1050,11 +1084,24 @@ void tc_set_trace(unsigned long long *buffer, int cta)
     g_trace_cta = cta;
 }
 
+// Query heads per sub-unit: the most heads of a KV group (a divisor of G) whose stacked rows
+// still fit one accumulator and the lse stager.
+int tc_gsub(const Geometry &g)
+{
+    const int cap = kEpiWG * kMaxGroups * 16 < 32 * kRowsPerLane ? kEpiWG * kMaxGroups * 16
+                                                                 : 32 * kRowsPerLane;
+    for (int gs = g.G; gs >= 1; --gs)
+        if (g.G % gs == 0 && gs * g.m <= cap)
+            return gs;
+    return 0;
+}
+
 bool tc_supported(const Geometry &g)
 {
-    if (g.variant != DGE_VARIANT_SCORED || (g.d != 64 && g.d != 128) ||
-        g.R > kEpiWG * kMaxGroups * 16 || g.R > 32 * kRowsPerLane ||
-        (size_t)((g.R + 3) & ~3) * 4 > (size_t)kStageBytes || g.m > 256 || g.G > 256)
+    if (g.variant != DGE_VARIANT_SCORED || (g.d != 64 && g.d != 128) || g.m > 256 || g.G > 256)
+        return false;
+    const int gs = tc_gsub(g);
+    if (gs == 0 || (size_t)((gs * g.m + 3) & ~3) * 4 > (size_t)kStageBytes)
         return false;
     int dev = 0, major = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -1066,8 +1113,11 @@ bool tc_supported(const Geometry &g)
 TcPlan tc_plan(const Geometry &g)
 {
     TcPlan p;
-    p.r_pad = (g.R + 15) & ~15;
-    p.r4 = (g.R + 3) & ~3;
+    p.gsub = tc_gsub(g);
+    p.nrb = p.gsub > 0 ? g.G / p.gsub : 1;
+    p.rows = p.gsub * g.m;
+    p.r_pad = (p.rows + 15) & ~15;
+    p.r4 = (p.rows + 3) & ~3;
     p.nslab = g.d / 64;
     // Key chunk (one task): as long as the phase-1 data of the tasks between an item's two
     // phases still fits in L2, i.e. (S + nchunks) chunks of K rows <= L2, which is about
@@ -1105,7 +1155,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
 {
     CUtensorMap tmK, tmQ;
     *encoded = encode_5d(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d, kTile, 1) &&
-               encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.m, g.d, g.m, g.G);
+               encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.m, g.d, g.m, plan.gsub);
     if (!*encoded)
         return cudaSuccess;
     int dev = 0, sms = 0;
@@ -1117,6 +1167,9 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
 
     TcArgs a;
     a.g = g;
+    a.rows = plan.rows;
+    a.nrb = plan.nrb;
+    a.gsub = plan.gsub;
     a.r_pad = plan.r_pad;
     a.r4 = plan.r4;
     a.acc_stride = (plan.r_pad + 31) & ~31;
@@ -1129,7 +1182,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
         // One pass, nothing to keep in L2: tasks of up to 32 tiles.
         a.nchunks = (a.unit_tiles + 31) / 32;
     }
-    a.items = g.U * a.nchunks;
+    a.items = g.U * a.nrb * a.nchunks;
     const int NG = plan.r_pad / 16;
     for (int w = 0, base = 0; w < kEpiWG; ++w) {
         a.ng[w] = NG / kEpiWG + (w < NG % kEpiWG ? 1 : 0);
@@ -1143,6 +1196,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.part = buf.part;
     a.lse2 = buf.lse2;
     a.raw = buf.raw;
+    a.raw_fx = plan.nrb > 1 ? buf.raw_fx : nullptr;
     a.count = buf.count;
     a.ready = buf.ready;
     a.status = buf.status;
@@ -1150,8 +1204,10 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.trace = g_trace;
     a.trace_cta = g_trace_cta;
 
+    // The traced build covers whole units only; row blocks run untraced.
     void (*kernel)(const CUtensorMap, const CUtensorMap, const TcArgs) =
-        a.trace ? score_tc_kernel<true> : score_tc_kernel<false>;
+        plan.nrb > 1 ? score_tc_kernel<false, true>
+                     : (a.trace ? score_tc_kernel<true, false> : score_tc_kernel<false, false>);
     err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                (int)plan.smem);
     if (err != cudaSuccess)
