@@ -313,7 +313,51 @@ bool want_tc(const Geometry &g)
     const char *env = getenv("DGE_SCORE_KERNEL");
     if (env && strcmp(env, "mma") == 0)
         return false;
-    return tc_supported(g);
+    return g.variant == DGE_VARIANT_H2O ? h2o_tc_supported(g) : tc_supported(g);
+}
+
+// H2O on the tensor cores: phase 1 (unless the normalisers are supplied: lse2 already holds
+// them), phase 2, then the warp-level kernels for units whose row sums left fp32's range.
+// False when the tensors cannot be described to TMA (nothing launched: use the warp path).
+int run_h2o_tc(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void *ws,
+               cudaStream_t stream, bool supplied, float *lse_out, bool *done)
+{
+    const Geometry &g = plan.g;
+    const H2oPlan hp = h2o_tc_plan(g);
+    float2 *partial = ws_at<float2>(ws, plan.off_partial);
+    float *lse2 = ws_at<float>(ws, plan.off_lse);
+    float *raw = ws_at<float>(ws, plan.off_raw);
+    uint32_t *ready = ws_at<uint32_t>(ws, plan.off_ready);
+    uint32_t *status = static_cast<uint32_t *>(ws);
+    bool encoded = false;
+    *done = false;
+    if (!supplied) {
+        DGE_CHECK_CUDA(cudaMemsetAsync(ready, 0, (size_t)g.U * sizeof(uint32_t), stream),
+                       "flag clear");
+        DGE_LAUNCH("h2o_tc_lse", stream,
+                   launch_h2o_tc(1, K, Q, g, hp, lse2, raw, ready, status, stream, &encoded));
+        if (!encoded)
+            return DGE_OK;
+    }
+    DGE_LAUNCH("h2o_tc_colsum", stream,
+               launch_h2o_tc(2, K, Q, g, hp, lse2, raw, ready, status, stream, &encoded));
+    if (!encoded)
+        return DGE_OK;
+    *done = true;
+    if (supplied)
+        return DGE_OK;
+    DGE_LAUNCH("recompute_lse", stream,
+               launch_lse_partial(K, Q, g, plan.rows_per_block, plan.chunk_keys, partial, stream,
+                                  ready));
+    DGE_LAUNCH("recompute_combine", stream,
+               launch_combine_lse(partial, g.U * g.R, plan.nchunks, lse2, stream, ready, g.R));
+    DGE_LAUNCH("recompute_colsum", stream,
+               launch_colsum_keys(K, Q, g, lse2, raw, stream, ready));
+    if (lse_out)
+        DGE_LAUNCH("lse_export", stream,
+                   launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
+                                     stream));
+    return DGE_OK;
 }
 
 // raw scores of every unit into the workspace.  lse_in (nullable): the caller's natural-log
@@ -354,6 +398,12 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
             }
         }
         DGE_LAUNCH("lse_import", stream, launch_lse_import(lse_in, lse2, g.U * g.R, stream));
+        if (g.variant == DGE_VARIANT_H2O && want_tc(g)) {
+            bool done = false;
+            const int rc = run_h2o_tc(plan, K, Q, ws, stream, true, nullptr, &done);
+            if (rc != DGE_OK || done)
+                return rc;
+        }
         if (g.variant == DGE_VARIANT_H2O)
             DGE_LAUNCH("colsum_keys", stream, launch_colsum_keys(K, Q, g, lse2, raw, stream));
         else
@@ -409,6 +459,12 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
                                              unit_flag, g.U, g.R, plan.tc.rows, lse_out, stream));
             return DGE_OK;
         }
+    }
+    if (g.variant == DGE_VARIANT_H2O && want_tc(g)) {
+        bool done = false;
+        const int rc = run_h2o_tc(plan, K, Q, ws, stream, false, lse_out, &done);
+        if (rc != DGE_OK || done)
+            return rc;
     }
     DGE_LAUNCH("lse_partial", stream, launch_lse_partial(K, Q, g, plan.rows_per_block, plan.chunk_keys, partial,
                                       stream));

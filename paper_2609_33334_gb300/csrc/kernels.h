@@ -47,7 +47,27 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
                             const TcPlan &plan, const TcBuffers &buf, cudaStream_t stream,
                             bool *encoded);
 cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
-                               const float *lse2, float *raw, cudaStream_t stream);
+                               const float *lse2, float *raw, cudaStream_t stream,
+                               const uint32_t *only = nullptr);
+
+// H2O scoring on the tcgen05 path (h2o_tc.cu): query blocks of pb positions x G heads.
+struct H2oPlan {
+    int pb;            // positions per query block
+    int rows;          // G * pb stacked rows of a block
+    int r_pad;         // rows rounded up to 16 (the MMA's N)
+    int nslab;         // d / 64
+    int nqb;           // query blocks per unit
+    int nkt;           // 128-key tiles of past keys per unit
+    size_t smem[2];    // dynamic shared memory of phase 1 / phase 2
+};
+bool h2o_tc_supported(const Geometry &g);
+H2oPlan h2o_tc_plan(const Geometry &g);
+// phase 1: lse2 [U][R] (base 2) and ready [U] (2 = recompute; zero before the launch);
+// phase 2: raw [U][P] from lse2.  *encoded is false when the tensors cannot be described to
+// TMA (nothing is launched then).
+cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                          const H2oPlan &plan, float *lse2, float *raw, uint32_t *ready,
+                          uint32_t *status, cudaStream_t stream, bool *encoded);
 
 // Pooling, selection, gather (select_compact.cu).
 cudaError_t launch_pool(const float *raw, float *out, int64_t U, int P, int pool, int kernel,

@@ -351,13 +351,16 @@ colsum_rows_kernel(TensorDesc K, TensorDesc Q, Geometry g, int chunk_keys, int n
 template <int D>
 __global__ void __launch_bounds__(kThreads)
 colsum_keys_kernel(TensorDesc K, TensorDesc Q, Geometry g, int nkb,
-                   const float *__restrict__ lse2, float *__restrict__ raw)
+                   const float *__restrict__ lse2, float *__restrict__ raw,
+                   const uint32_t *__restrict__ only)
 {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ float sL[2][kRowTile];
     __shared__ int sPos[2][kRowTile];
     const int64_t u = blockIdx.x / nkb;
     const int kb = (int)(blockIdx.x % nkb);
+    if (only && only[u] != kUnitRecompute)
+        return;
     int l, bb, h;
     unit_coords(g, u, l, bb, h);
     const int k_lo = kb * kKeyBlock;
@@ -547,7 +550,8 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
 }
 
 cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
-                               const float *lse2, float *raw, cudaStream_t stream)
+                               const float *lse2, float *raw, cudaStream_t stream,
+                               const uint32_t *only)
 {
     const int nkb = (g.P + kKeyBlock - 1) / kKeyBlock;
     const int64_t blocks = g.U * nkb;
@@ -558,14 +562,14 @@ cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const G
         if (err != cudaSuccess)
             return err;
         colsum_keys_kernel<128><<<(unsigned)blocks, kThreads, smem, stream>>>(K, Q, g, nkb, lse2,
-                                                                              raw);
+                                                                              raw, only);
     } else {
         const size_t smem = (size_t)(kKeyBlock + 2 * kRowTile) * Pad<64>::kStride * 2;
         err = prepare(colsum_keys_kernel<64>, smem);
         if (err != cudaSuccess)
             return err;
         colsum_keys_kernel<64><<<(unsigned)blocks, kThreads, smem, stream>>>(K, Q, g, nkb, lse2,
-                                                                             raw);
+                                                                             raw, only);
     }
     return cudaGetLastError();
 }

@@ -32,6 +32,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "tc_common.cuh"
 #include "tc_ptx.cuh"
 
 namespace dge {
@@ -65,7 +66,7 @@ constexpr int kCtrlBytes = 400;            // barriers, TMEM address, flags (16-
 constexpr int kRowsPerLane = 5;           // rows of the lse merge per lane (R <= 160)
 // Flag slots (ints): abort, then the parity of the last arm of every key stage, query
 // buffer and the staging buffer (-1 = never armed) for the drain.
-constexpr int kFlagAbort = 0, kFlagKArm = 4, kFlagQArm = 8, kFlagSArm = 10;
+constexpr int kFlagAbort = tc::kFlagAbort, kFlagKArm = 4, kFlagQArm = 8, kFlagSArm = 10;
 
 struct TcArgs {
     Geometry g;
@@ -222,80 +223,16 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int ks
     return s;
 }
 
-// Bounded wait on an mbarrier phase.  Returns false when the CTA has aborted or the
-// wait outlived the timeout (then it aborts the CTA and records the status).
-__device__ bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *flag, const TcArgs &a)
+// Bounded wait on an mbarrier phase (false once the CTA has aborted or timed out).
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *flag,
+                                         const TcArgs &a)
 {
-    uint64_t t0 = 0;
-    uint32_t spins = 0;
-    while (!ptx::mbar_try_wait(bar, parity)) {
-        if ((++spins & 63) == 0) {
-            if (flag[kFlagAbort])
-                return false;
-            const uint64_t now = ptx::globaltimer();
-            if (t0 == 0) {
-                t0 = now;
-            } else if (now - t0 > a.timeout_ns) {
-                flag[kFlagAbort] = 1;
-                set_status(a.status, DGE_ERR_DEVICE_TIMEOUT);
-                return false;
-            }
-        }
-    }
-    return true;
+    return tc::wait_bar(bar, parity, flag, a.timeout_ns, a.status);
 }
 
-// Bounded wait that ignores the abort flag (teardown drains).
-__device__ void drain_bar(uint64_t *bar, uint32_t parity, unsigned long long limit_ns)
-{
-    const uint64_t t0 = ptx::globaltimer();
-    while (!ptx::mbar_try_wait(bar, parity))
-        if (ptx::globaltimer() - t0 > limit_ns)
-            return;
-}
-
-// In-place sums over the 32 lanes of a warp, for 32 per-lane values held as two
-// 16-value groups a (columns 0..15) and b (16..31): afterwards a[0] of lane l holds
-// the total of column l.  Each step halves the values a lane keeps: the lane whose
-// bit o is set keeps the upper half, its partner the lower half.
-__device__ __forceinline__ void transpose_sum32(float (&a)[16], float (&b)[16], int lane)
-{
-    const bool up16 = (lane & 16) != 0;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const float send = up16 ? a[i] : b[i];
-        const float keep = up16 ? b[i] : a[i];
-        a[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
-    }
-#pragma unroll
-    for (int o = 8; o >= 1; o >>= 1) {
-        const bool upper = (lane & o) != 0;
-#pragma unroll
-        for (int i = 0; i < o; ++i) {
-            const float send = upper ? a[i] : a[i + o];
-            const float keep = upper ? a[i + o] : a[i];
-            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-        }
-    }
-}
-
-// Same for one 16-value group: lanes l and l ^ 16 both end with column l & 15 in a[0].
-__device__ __forceinline__ void transpose_sum16(float (&a)[16], int lane)
-{
-#pragma unroll
-    for (int i = 0; i < 16; ++i)
-        a[i] += __shfl_xor_sync(0xffffffffu, a[i], 16);
-#pragma unroll
-    for (int o = 8; o >= 1; o >>= 1) {
-        const bool upper = (lane & o) != 0;
-#pragma unroll
-        for (int i = 0; i < o; ++i) {
-            const float send = upper ? a[i] : a[i + o];
-            const float keep = upper ? a[i + o] : a[i];
-            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-        }
-    }
-}
+using tc::drain_bar;
+using tc::transpose_sum16;
+using tc::transpose_sum32;
 
 // Visibility of the 16 columns cb .. cb+15 to `key` on tiles that reach the observation
 // rows' own positions: row r sits at first_causal + r % m and sees keys up to there.
@@ -1031,12 +968,19 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         ptx::tmem_dealloc(tmem_base, kTmemCols);
 }
 
+unsigned long long *g_trace = nullptr;
+int g_trace_cta = 0;
+
+}  // namespace
+
+namespace tc {
+
 using Encode = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
                             const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
                             const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
                             CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-Encode encode_fn()
+Encode encode_fn_impl()
 {
     static Encode fn = nullptr;
     static bool tried = false;
@@ -1052,11 +996,10 @@ Encode encode_fn()
     return fn;
 }
 
-// 5-D map over [L][b][heads][rows][d] with box {64, box_rows, box_heads, 1, 1}.
 bool encode_5d(CUtensorMap *map, const TensorDesc &t, int L, int b, int heads, int rows, int d,
                int box_rows, int box_heads)
 {
-    Encode fn = encode_fn();
+    Encode fn = encode_fn_impl();
     if (!fn)
         return false;
     const cuuint64_t dims[5] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)heads, (cuuint64_t)b,
@@ -1073,10 +1016,12 @@ bool encode_5d(CUtensorMap *map, const TensorDesc &t, int L, int b, int heads, i
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-unsigned long long *g_trace = nullptr;
-int g_trace_cta = 0;
+bool have_tensor_maps()
+{
+    return encode_fn_impl() != nullptr;
+}
 
-}  // namespace
+}  // namespace tc
 
 void tc_set_trace(unsigned long long *buffer, int cta)
 {
@@ -1107,7 +1052,7 @@ bool tc_supported(const Geometry &g)
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess)
         return false;
-    return major == 10 && encode_fn() != nullptr;
+    return major == 10 && tc::have_tensor_maps();
 }
 
 TcPlan tc_plan(const Geometry &g)
@@ -1154,8 +1099,8 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
                             bool *encoded)
 {
     CUtensorMap tmK, tmQ;
-    *encoded = encode_5d(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d, kTile, 1) &&
-               encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.m, g.d, g.m, plan.gsub);
+    *encoded = tc::encode_5d(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d, kTile, 1) &&
+               tc::encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.m, g.d, g.m, plan.gsub);
     if (!*encoded)
         return cudaSuccess;
     int dev = 0, sms = 0;

@@ -1,0 +1,100 @@
+// tc_common.cuh -- device helpers shared by the tcgen05 kernels (score_tc.cu, h2o_tc.cu):
+// bounded mbarrier waits and the warp transpose-and-add used to reduce per-lane row sums.
+#pragma once
+
+#include <cuda.h>
+
+#include "common.cuh"
+#include "tc_ptx.cuh"
+
+namespace dge {
+namespace tc {
+
+// Slot 0 of a kernel's shared flag block: set once the CTA has aborted.
+constexpr int kFlagAbort = 0;
+
+// Bounded wait on an mbarrier phase.  Returns false when the CTA has aborted or the wait
+// outlived `timeout_ns` (then it aborts the CTA and records DGE_ERR_DEVICE_TIMEOUT).
+__device__ inline bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *flag,
+                                unsigned long long timeout_ns, uint32_t *status)
+{
+    uint64_t t0 = 0;
+    uint32_t spins = 0;
+    while (!ptx::mbar_try_wait(bar, parity)) {
+        if ((++spins & 63) == 0) {
+            if (flag[kFlagAbort])
+                return false;
+            const uint64_t now = ptx::globaltimer();
+            if (t0 == 0) {
+                t0 = now;
+            } else if (now - t0 > timeout_ns) {
+                flag[kFlagAbort] = 1;
+                set_status(status, DGE_ERR_DEVICE_TIMEOUT);
+                return false;
+            }
+        }
+    }
+    return true;
+}
+
+// Bounded wait that ignores the abort flag (teardown drains).
+__device__ inline void drain_bar(uint64_t *bar, uint32_t parity, unsigned long long limit_ns)
+{
+    const uint64_t t0 = ptx::globaltimer();
+    while (!ptx::mbar_try_wait(bar, parity))
+        if (ptx::globaltimer() - t0 > limit_ns)
+            return;
+}
+
+// In-place sums over the 32 lanes of a warp, for 32 per-lane values held as two
+// 16-value groups a (columns 0..15) and b (16..31): afterwards a[0] of lane l holds
+// the total of column l.  Each step halves the values a lane keeps: the lane whose
+// bit o is set keeps the upper half, its partner the lower half.
+__device__ __forceinline__ void transpose_sum32(float (&a)[16], float (&b)[16], int lane)
+{
+    const bool up16 = (lane & 16) != 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const float send = up16 ? a[i] : b[i];
+        const float keep = up16 ? b[i] : a[i];
+        a[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+    }
+#pragma unroll
+    for (int o = 8; o >= 1; o >>= 1) {
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < o; ++i) {
+            const float send = upper ? a[i] : a[i + o];
+            const float keep = upper ? a[i + o] : a[i];
+            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+}
+
+// Same for one 16-value group: lanes l and l ^ 16 both end with column l & 15 in a[0].
+__device__ __forceinline__ void transpose_sum16(float (&a)[16], int lane)
+{
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+        a[i] += __shfl_xor_sync(0xffffffffu, a[i], 16);
+#pragma unroll
+    for (int o = 8; o >= 1; o >>= 1) {
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < o; ++i) {
+            const float send = upper ? a[i] : a[i + o];
+            const float keep = upper ? a[i + o] : a[i];
+            a[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+}
+
+// Host: a 5-D TMA map over [L][b][heads][rows][d] (bf16, 128-byte swizzle) with box
+// {64, box_rows, box_heads, 1, 1}; false when the driver entry point is missing or the strides
+// are not 16-byte multiples.
+bool encode_5d(CUtensorMap *map, const TensorDesc &t, int L, int b, int heads, int rows, int d,
+               int box_rows, int box_heads);
+bool have_tensor_maps();
+
+}  // namespace tc
+}  // namespace dge

@@ -21,7 +21,7 @@ CASES = {
     "c3_small": WL["c3_8b_32k_pyramid"].with_(L=2, b=2, n=4500, budgets=(900, 610),
                                               n_spans=8),
     "c1_tiny": WL["c1_tiny"],
-    "c4_small": WL["c4_h2o_8k"].with_(L=1, b=2, n=1000, budgets=(200,)),   # H2O, warp level
+    "c4_small": WL["c4_h2o_8k"].with_(L=1, b=2, n=1000, budgets=(200,)),   # H2O
     "c5_small": WL["c5_70b_128k"].with_(L=1, n=3000, budgets=(700,), n_spans=8),  # R = 528
 }
 

@@ -72,6 +72,11 @@ SMALL = {
     "max_pool_3_d128": WL["c1_tiny"].with_(d=128, pool_kernel=3),
     "gqa8_ragged": WL["c1_tiny"].with_(Hq=16, Hkv=2, n=2117, budgets=(333,)),
     "h2o_tiny": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=4, Hkv=2, d=64, n=300, budgets=(100,)),
+    # H2O query blocks: G = 5 gives 28 positions x 5 heads = 140 rows (4 padded columns),
+    # G = 8 gives 18 positions, G = 1 a single 144-position block of one head
+    "h2o_g5_padded": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=10, Hkv=2, d=64, n=777, budgets=(200,)),
+    "h2o_g8": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=16, Hkv=2, n=500, budgets=(150,)),
+    "h2o_g1": WL["c4_h2o_8k"].with_(L=2, b=1, Hq=2, Hkv=2, n=403, budgets=(120, 90)),
     "slm_keep_all": WL["c5_slm"].with_(L=1, n=300, Hq=8, Hkv=2, budgets=(300,), n_spans=0),
 }
 
@@ -225,14 +230,16 @@ def _kernels_run(fn):
     return {name for name, _, _ in B.dge_profile_end()}
 
 
-@pytest.mark.parametrize("name,expect_tc", [("c2_small", True), ("c1_tiny", True),
-                                            ("c5_small", True), ("c4_small", False)])
-def test_tensor_core_path_is_taken_where_eligible(name, expect_tc):
+@pytest.mark.parametrize("name,kernel", [("c2_small", "score_tc"), ("c1_tiny", "score_tc"),
+                                         ("c5_small", "score_tc"), ("c4_small", "h2o_tc_colsum"),
+                                         ("h2o_g8", "h2o_tc_colsum")])
+def test_tensor_core_path_is_taken_where_eligible(name, kernel):
     wl = SMALL.get(name) or WL[name]
     tens = inputs.make_inputs(wl, device="cuda")
     p = api.problem_from_workload(wl)
     names = _kernels_run(lambda: api.evict(p, tens["K"], tens["V"], tens["Q"]))
-    assert ("score_tc" in names) == expect_tc, names
+    assert kernel in names, names
+    assert "colsum_rows" not in names and "colsum_keys" not in names, names
 
 
 def test_paths_agree_closely():
@@ -271,6 +278,36 @@ def test_row_blocks_are_deterministic_and_agree_with_warp_level_path():
     assert torch.equal(a, a2)
     rel = ((a - b).abs() / b.abs().clamp_min(1e-6 * b.abs().max())).max().item()
     assert rel < 1e-4, rel
+
+
+def test_h2o_paths_agree_and_repeat():
+    """H2O on tcgen05 (query blocks, fp32 sums without a running maximum) agrees with the
+    warp-level kernels far inside the oracle tolerance, and re-runs are byte-identical."""
+    import os
+    wl = SMALL["c4_small"]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    a = api.score(p, tens["K"], tens["Q"])
+    a2 = api.score(p, tens["K"], tens["Q"])
+    os.environ["DGE_SCORE_KERNEL"] = "mma"
+    try:
+        b = api.score(p, tens["K"], tens["Q"])
+    finally:
+        del os.environ["DGE_SCORE_KERNEL"]
+    torch.cuda.synchronize()
+    assert torch.equal(a, a2)
+    rel = ((a - b).abs() / b.abs().clamp_min(1e-6 * b.abs().max())).max().item()
+    assert rel < 1e-4, rel
+
+
+def test_h2o_large_logits_are_recomputed_exactly():
+    """H2O units whose fp32 row sums leave range are flagged by the tensor-core kernel and
+    recomputed by the warp-level kernels (which carry a running maximum)."""
+    wl = SMALL["c4_small"].with_(b=1)
+    tens = inputs.make_inputs(wl, device="cuda")
+    tens["Q"] = (tens["Q"].float() * 24.0).to(torch.bfloat16)
+    tens, out = run(wl, tens=tens)
+    check_all(wl, tens, out)
 
 
 def test_large_logits_are_recomputed_exactly():
