@@ -52,7 +52,11 @@ constexpr int kAccBufs = 3;               // TMEM accumulators
 constexpr int kTmemCols = 512;
 constexpr int kKSlab = kTile * 128;       // 128 keys x 64 bf16
 constexpr int kXchBufs = 4;               // phase-2 end-of-task exchange areas
-constexpr int kLseStride = 256;           // floats per staged -lse block
+// -lse of the streamed query blocks, staged kLseGroup blocks at a time into one of two slots:
+// a hand-off (one wait, one arrival) every kLseGroup tiles rather than every tile.
+constexpr int kLseGroup = 4;
+constexpr int kLseSlots = 2;
+constexpr int kLseBlock = 160;            // floats per block (>= rows, 16-byte multiple)
 constexpr int kLseLoads = (kMaxBlockRows + 31) / 32;   // staged rows per lane
 constexpr uint32_t kReadyBad = 2;
 
@@ -100,7 +104,7 @@ __host__ __device__ inline size_t smem_bytes(int phase, int r_pad, int nslab)
     return 1024                                                 // alignment slack
            + (size_t)2 * nslab * stat_slab(phase, r_pad)        // stationary operand
            + (size_t)kStages * nslab * ring_slab(phase, r_pad)  // streamed operand
-           + kCtrlBytes + (size_t)kStages * kLseStride * 4
+           + kCtrlBytes + (size_t)kLseSlots * kLseGroup * kLseBlock * 4
            + (size_t)2 * kEpiWG * 4 * kMaxGroups * 16 * 4 + (size_t)kXchBufs * kEpiWG * kTile * 4;
 }
 
@@ -110,7 +114,7 @@ struct Smem {
     uint64_t *bar;     // [kNumBars]
     uint32_t *tmem;    // allocation result
     int *flag;         // [16]
-    float *lse;        // [kStages][kLseStride] -lse of the streamed blocks (phase 2)
+    float *lse;        // [kLseSlots][kLseGroup][kLseBlock] -lse of streamed blocks (phase 2)
     float *red;        // [2][kEpiWG][4][kMaxGroups * 16] per-warp row sums (phase 1)
     float *xch;        // [kXchBufs][kEpiWG][128] per-warpgroup column sums (phase 2)
 };
@@ -129,7 +133,7 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int phase, int r_pad, int ns
     s.flag = reinterpret_cast<int *>(raw + off + kNumBars * 8 + 16);
     off += kCtrlBytes;
     s.lse = reinterpret_cast<float *>(raw + off);
-    off += kStages * kLseStride * 4;
+    off += kLseSlots * kLseGroup * kLseBlock * 4;
     s.red = reinterpret_cast<float *>(raw + off);
     off += 2 * kEpiWG * 4 * kMaxGroups * 16 * 4;
     s.xch = reinterpret_cast<float *>(raw + off);
@@ -260,6 +264,8 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
         for (int i = 0; i < kStages; ++i) {
             ptx::mbar_init(&sm.bar[kBarRingFull + i], 1);
             ptx::mbar_init(&sm.bar[kBarRingEmpty + i], 1);
+        }
+        for (int i = 0; i < kLseSlots; ++i) {
             ptx::mbar_init(&sm.bar[kBarLseFull + i], 1);
             ptx::mbar_init(&sm.bar[kBarLseEmpty + i], kEpiWarps);
         }
@@ -448,8 +454,7 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
             };
             if (warp == 2 && a.phase == 2) {
                 // ---- -lse of every streamed query block, per row: -inf past the cache ------
-                int ls = 0;
-                uint32_t lph = 0;
+                int64_t nb = 0;      // blocks staged so far: slot (nb / kLseGroup) % kLseSlots
                 int hd[kLseLoads];   // query head of each of this lane's rows
 #pragma unroll
                 for (int j = 0; j < kLseLoads; ++j)
@@ -458,11 +463,14 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                     Task T;
                     get_task(a, item, T);
                     const float *src = a.lse2 + T.u * g.R;
-                    for (int i = 0; i < T.ntiles; ++i) {
-                        if (!wait_w(&sm.bar[kBarLseEmpty + ls], lph ^ 1))
+                    for (int i = 0; i < T.ntiles; ++i, ++nb) {
+                        const int sub = (int)(nb % kLseGroup);
+                        const int slot = (int)((nb / kLseGroup) % kLseSlots);
+                        const uint32_t lph = (uint32_t)((nb / (kLseGroup * kLseSlots)) & 1);
+                        if (sub == 0 && !wait_w(&sm.bar[kBarLseEmpty + slot], lph ^ 1))
                             break;
                         const int p0 = (T.first + i) * a.pb;
-                        float *L = sm.lse + ls * kLseStride;
+                        float *L = sm.lse + (slot * kLseGroup + sub) * kLseBlock;
                         // All of a lane's loads in flight at once: one L2 round trip a block.
                         float v[kLseLoads];
 #pragma unroll
@@ -478,14 +486,19 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                         for (int j = 0; j < kLseLoads; ++j)
                             if (lane + 32 * j < a.r_pad)
                                 L[lane + 32 * j] = v[j];
-                        __syncwarp();
-                        if (lane == 0)
-                            ptx::mbar_arrive(&sm.bar[kBarLseFull + ls]);
-                        if (++ls == kStages) {
-                            ls = 0;
-                            lph ^= 1;
+                        if (sub == kLseGroup - 1) {
+                            __syncwarp();
+                            if (lane == 0)
+                                ptx::mbar_arrive(&sm.bar[kBarLseFull + slot]);
                         }
                     }
+                }
+                // A last, partly filled group.
+                if (!dead && nb % kLseGroup != 0) {
+                    __syncwarp();
+                    if (lane == 0)
+                        ptx::mbar_arrive(
+                            &sm.bar[kBarLseFull + (int)((nb / kLseGroup) % kLseSlots)]);
                 }
             } else if (warp == 3 && a.phase == 1) {
                 // ---- row sums of a query block -> lse_r ---------------------------------------
@@ -628,8 +641,9 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                 }
             }
         } else {
-            int ls = 0, xc = 0;
-            uint32_t lph = 0;
+            int xc = 0;
+            int64_t nb = 0;      // streamed blocks so far (the stager's count)
+            bool lse_ok = false;
             for (int64_t item = blockIdx.x; item < a.items; item += S) {
                 Task T;
                 get_task(a, item, T);
@@ -642,9 +656,15 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                     const int p0 = (T.first + i) * a.pb;
                     const bool diag = p0 < k0 + kTile;  // some row precedes some key
                     float nL[kMaxGroups][16];
-                    if (wait_uniform(&sm.bar[kBarLseFull + ls], lph)) {
-                        const float4 *L4 =
-                            reinterpret_cast<const float4 *>(sm.lse + ls * kLseStride + col_base);
+                    const int sub = (int)(nb % kLseGroup);
+                    const int slot = (int)((nb / kLseGroup) % kLseSlots);
+                    if (sub == 0)
+                        lse_ok = wait_uniform(&sm.bar[kBarLseFull + slot],
+                                              (uint32_t)((nb / (kLseGroup * kLseSlots)) & 1));
+                    ++nb;
+                    if (lse_ok) {
+                        const float4 *L4 = reinterpret_cast<const float4 *>(
+                            sm.lse + (slot * kLseGroup + sub) * kLseBlock + col_base);
 #pragma unroll
                         for (int gi = 0; gi < kMaxGroups; ++gi)
 #pragma unroll
@@ -657,19 +677,17 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                                 nL[gi][4 * q + 2] = f.z;
                                 nL[gi][4 * q + 3] = f.w;
                             }
-                        __syncwarp();
-                        if (lane == 0)
-                            ptx::mbar_arrive(&sm.bar[kBarLseEmpty + ls]);
+                        if (sub == kLseGroup - 1) {
+                            __syncwarp();
+                            if (lane == 0)
+                                ptx::mbar_arrive(&sm.bar[kBarLseEmpty + slot]);
+                        }
                     } else {
 #pragma unroll
                         for (int gi = 0; gi < kMaxGroups; ++gi)
 #pragma unroll
                             for (int c = 0; c < 16; ++c)
                                 nL[gi][c] = -INFINITY;
-                    }
-                    if (++ls == kStages) {
-                        ls = 0;
-                        lph ^= 1;
                     }
                     if (acquire_acc(ab, aph)) {
                         const uint32_t tbase =

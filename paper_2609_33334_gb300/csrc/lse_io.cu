@@ -57,7 +57,7 @@ __global__ void fixed_to_float_kernel(const unsigned long long *__restrict__ fx,
 {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (int64_t)gridDim.x * blockDim.x)
-        out[i] = (float)((double)(long long)fx[i] * 0x1p-40);
+        out[i] = __ll2float_rn((long long)fx[i]) * 0x1p-40f;   // one rounding, exact scaling
 }
 
 // A unit is recomputed when any of its row blocks left fp32's range.
