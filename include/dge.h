@@ -108,6 +108,35 @@ typedef struct dge_tensor {
     int64_t stride_layer, stride_batch, stride_head, stride_pos;
 } dge_tensor;
 
+/*
+ * A paged KV cache (block table), the layout paged-attention serving engines keep (the paper
+ * names paged-attention batching as the route to throughput, Sec. "Limitations"): every
+ * layer's K (and V) lives in a pool of fixed-size pages, and a sequence's positions are the
+ * concatenation of the pages its block table lists.  With paging, the dge_tensor of K and of
+ * V describes its pools: data = slot 0 of page 0 of layer 0's pool, stride_layer = elements
+ * between the layers' pools, stride_head = between the KV heads of a slot, stride_pos = between
+ * the slots of a page (stride_batch is unused); position p of sequence b is slot
+ * p % page_size of page block_table[b * pages_per_seq + p / page_size].  K and V share the
+ * block table and the page geometry.  Q is never paged.
+ *   block_table: device int32 [b][pages_per_seq], 4-byte aligned; the entries covering
+ *     positions [0, n) must lie in [0, num_pages) (an entry outside is read as page 0);
+ *   page_size: 16, 32 or 64, or a multiple of 128;
+ *   pages_per_seq >= ceil(n / page_size); num_pages >= 1 (pages in each layer's pool);
+ *   stride_page: elements between pages, a positive multiple of 8.
+ * Every call that takes K / V accepts it: scoring reads the pages (one TMA box per page of a
+ * 128-key tile), the packed gather reads them, the in-place gather moves row r of every
+ * unit to position r of the same sequence's pages (so its first ceil(B / page_size) pages
+ * hold the kept cache and the rest can be returned to the pool).
+ */
+typedef struct dge_paging {
+    const int32_t *block_table;
+    int32_t page_size;
+    int32_t pages_per_seq;
+    int32_t num_pages;
+    int32_t reserved;     /* 0 */
+    int64_t stride_page;
+} dge_paging;
+
 /* Inputs and outputs of dge_evict / dge_score. */
 typedef struct dge_buffers {
     dge_tensor K;        /* [L][b][Hkv][n][d] */
@@ -132,6 +161,8 @@ typedef struct dge_buffers {
      * computed.  Both 4-byte aligned; NULL to leave unused. */
     const float *lse_in;
     float *lse_out;
+    /* K and V as a paged cache (NULL: the [L][b][Hkv][n][d] layout above); see dge_paging. */
+    const dge_paging *paging;
 } dge_buffers;
 
 /*
@@ -201,6 +232,11 @@ int dge_select(const dge_problem *p, const float *scores, int32_t *idx, void *st
 int dge_compact(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
                 const dge_tensor *V, void *Kc, void *Vc, void *ws, void *stream);
 
+/* dge_compact over a paged cache (K, V describe the pools; see dge_paging). */
+int dge_compact_paged(const dge_problem *p, const dge_paging *paging, const int32_t *idx,
+                      const dge_tensor *K, const dge_tensor *V, void *Kc, void *Vc, void *ws,
+                      void *stream);
+
 /*
  * The whole pass, score -> pool -> select -> compact, enqueued on one stream
  * with no host synchronisation.  Writes bufs->idx, Kc, Vc and, when not NULL,
@@ -221,6 +257,11 @@ int dge_evict(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
  */
 int dge_compact_inplace(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
                         const dge_tensor *V, void *ws, void *stream);
+
+/* dge_compact_inplace over a paged cache: row r of every unit moves to position r of the same
+ * sequence through the block table (see dge_paging). */
+int dge_compact_inplace_paged(const dge_problem *p, const dge_paging *paging, const int32_t *idx,
+                              const dge_tensor *K, const dge_tensor *V, void *ws, void *stream);
 
 /*
  * dge_evict with the in-place compaction: score -> pool -> select, then the kept rows move

@@ -5,6 +5,7 @@ in the library's CUDA kernels on the tensors' device and the current stream.
 """
 from __future__ import annotations
 
+import ctypes
 import dataclasses
 from typing import Optional, Sequence
 
@@ -69,6 +70,43 @@ class Problem:
         return offs
 
 
+@dataclasses.dataclass
+class Paging:
+    """A paged cache (dge_paging): K and V are then pools [L][num_pages][page_size][Hkv][d]
+    and position p of sequence b lives in slot p % page_size of page
+    block_table[b, p // page_size] (int32 [b][pages_per_seq] on the device)."""
+
+    block_table: torch.Tensor
+    page_size: int
+
+    def c(self, pool: torch.Tensor) -> B.dge_paging:
+        bt = self.block_table
+        if bt.dtype != torch.int32 or not bt.is_contiguous() or bt.dim() != 2:
+            raise ValueError("block_table must be a contiguous int32 [b][pages_per_seq] tensor")
+        if pool.dim() != 5 or pool.shape[2] != self.page_size:
+            raise ValueError("paged K / V must be [L][num_pages][page_size][Hkv][d]")
+        return B.dge_paging(block_table=bt.data_ptr(), page_size=self.page_size,
+                            pages_per_seq=bt.shape[1], num_pages=pool.shape[1],
+                            stride_page=pool.stride(1))
+
+
+def _kv_desc(t: torch.Tensor, paging: Optional[Paging]) -> B.dge_tensor:
+    if paging is None:
+        return B.tensor_desc(t)
+    if t.dim() != 5 or t.stride(-1) != 1:
+        raise ValueError("expected a 5-D pool with a contiguous last dim")
+    s = t.stride()   # [L][page][slot][head][d]
+    return B.dge_tensor(data=t.data_ptr(), stride_layer=s[0], stride_batch=0,
+                        stride_head=s[3], stride_pos=s[2])
+
+
+def _paging_ptr(paging: Optional[Paging], pool: torch.Tensor):
+    if paging is None:
+        return None, None
+    c = paging.c(pool)
+    return c, ctypes.pointer(c)
+
+
 def problem_from_workload(wl) -> Problem:
     """The Problem of a synthetic workload (``inputs.Workload``)."""
     return Problem(L=wl.L, b=wl.b, Hq=wl.Hq, Hkv=wl.Hkv, d=wl.d, n=wl.n, budgets=wl.budgets,
@@ -106,13 +144,14 @@ def _lse_arg(p: Problem, lse_in: Optional[torch.Tensor]) -> int:
 def evict(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torch.Tensor] = None, *,
           want_scores: bool = False, lse_in: Optional[torch.Tensor] = None,
           want_lse: bool = False, ws: Optional[torch.Tensor] = None,
-          out: Optional[dict] = None, stream=None) -> dict:
+          out: Optional[dict] = None, paging: Optional[Paging] = None, stream=None) -> dict:
     """dge_evict: the fused score -> pool -> select -> compact pass.
 
     Returns {"idx", "Kc", "Vc", "scores", "lse"} (scores / lse are None unless requested).
     ``lse_in``: the rows' natural-log normalisers [L][b][Hq][rows] (Problem.lse_shape), so the
     scoring reads K once; ``want_lse``: return the normalisers the scoring computed.
-    ``out`` may hold preallocated outputs with those keys.
+    ``out`` may hold preallocated outputs with those keys.  ``paging``: K and V are the pools
+    of a paged cache (see Paging).
     """
     _check_cache(K, "K")
     _check_cache(V, "V")
@@ -133,16 +172,18 @@ def evict(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torch.Tensor
     o.setdefault("lse", None)
     if ws is None:
         ws = workspace(p, dev)
-    bufs = B.dge_buffers(K=B.tensor_desc(K), V=B.tensor_desc(V), Q=B.tensor_desc(Q),
+    pg, pg_ptr = _paging_ptr(paging, K)
+    bufs = B.dge_buffers(K=_kv_desc(K, paging), V=_kv_desc(V, paging), Q=B.tensor_desc(Q),
                          scores=B.ptr(o["scores"]), idx=B.ptr(o["idx"]), Kc=B.ptr(o["Kc"]),
                          Vc=B.ptr(o["Vc"]), lse_in=_lse_arg(p, lse_in),
-                         lse_out=B.ptr(o["lse"]) if want_lse and lse_in is None else 0)
+                         lse_out=B.ptr(o["lse"]) if want_lse and lse_in is None else 0,
+                         paging=pg_ptr)
     B.dge_evict(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
     return o
 
 
 def score(p: Problem, K: torch.Tensor, Q: torch.Tensor, *, lse_in=None, want_lse=False,
-          ws=None, stream=None):
+          ws=None, paging: Optional[Paging] = None, stream=None):
     """dge_score: final (pooled) scores [unit][P] in float32.
 
     With ``want_lse`` returns (scores, lse); ``lse_in`` as for evict()."""
@@ -153,8 +194,9 @@ def score(p: Problem, K: torch.Tensor, Q: torch.Tensor, *, lse_in=None, want_lse
         if want_lse and lse_in is None else None
     if ws is None:
         ws = workspace(p, K.device)
-    bufs = B.dge_buffers(K=B.tensor_desc(K), Q=B.tensor_desc(Q), scores=scores.data_ptr(),
-                         lse_in=_lse_arg(p, lse_in), lse_out=B.ptr(lse))
+    pg, pg_ptr = _paging_ptr(paging, K)
+    bufs = B.dge_buffers(K=_kv_desc(K, paging), Q=B.tensor_desc(Q), scores=scores.data_ptr(),
+                         lse_in=_lse_arg(p, lse_in), lse_out=B.ptr(lse), paging=pg_ptr)
     B.dge_score(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
     return (scores, lse) if want_lse else scores
 
@@ -168,34 +210,45 @@ def select(p: Problem, scores: Optional[torch.Tensor], *, stream=None) -> torch.
 
 
 def compact(p: Problem, idx: torch.Tensor, K: torch.Tensor, V: torch.Tensor, *, ws=None,
-            stream=None) -> tuple:
-    """dge_compact: packed Kc, Vc gathered at idx."""
+            paging: Optional[Paging] = None, stream=None) -> tuple:
+    """dge_compact (dge_compact_paged with ``paging``): packed Kc, Vc gathered at idx."""
     _check_cache(K, "K")
     _check_cache(V, "V")
     rows = p.packed_rows()
     Kc = torch.empty((rows, p.d), dtype=torch.bfloat16, device=K.device)
     Vc = torch.empty_like(Kc)
-    kd, vd = B.tensor_desc(K), B.tensor_desc(V)
-    B.dge_compact(p.c(), idx.data_ptr(), kd, vd, Kc.data_ptr(), Vc.data_ptr(),
-                  B.ptr(ws), _stream(stream))
+    kd, vd = _kv_desc(K, paging), _kv_desc(V, paging)
+    if paging is None:
+        B.dge_compact(p.c(), idx.data_ptr(), kd, vd, Kc.data_ptr(), Vc.data_ptr(),
+                      B.ptr(ws), _stream(stream))
+    else:
+        B.dge_compact_paged(p.c(), paging.c(K), idx.data_ptr(), kd, vd, Kc.data_ptr(),
+                            Vc.data_ptr(), B.ptr(ws), _stream(stream))
     return Kc, Vc
 
 
 def compact_inplace(p: Problem, idx: torch.Tensor, K: torch.Tensor, V: torch.Tensor, *,
-                    ws=None, stream=None) -> None:
-    """dge_compact_inplace: rows [0, B_l) of every unit of K and V become the kept rows."""
+                    ws=None, paging: Optional[Paging] = None, stream=None) -> None:
+    """dge_compact_inplace: rows [0, B_l) of every unit of K and V become the kept rows (with
+    ``paging``: positions [0, B_l) of every sequence's pages)."""
     _check_cache(K, "K")
     _check_cache(V, "V")
-    B.dge_compact_inplace(p.c(), idx.data_ptr(), B.tensor_desc(K), B.tensor_desc(V),
-                          B.ptr(ws), _stream(stream))
+    if paging is None:
+        B.dge_compact_inplace(p.c(), idx.data_ptr(), B.tensor_desc(K), B.tensor_desc(V),
+                              B.ptr(ws), _stream(stream))
+    else:
+        B.dge_compact_inplace_paged(p.c(), paging.c(K), idx.data_ptr(), _kv_desc(K, paging),
+                                    _kv_desc(V, paging), B.ptr(ws), _stream(stream))
 
 
 def evict_inplace(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torch.Tensor] = None,
                   *, want_scores: bool = False, lse_in: Optional[torch.Tensor] = None,
                   want_lse: bool = False, ws: Optional[torch.Tensor] = None,
-                  out: Optional[dict] = None, stream=None) -> dict:
+                  out: Optional[dict] = None, paging: Optional[Paging] = None,
+                  stream=None) -> dict:
     """dge_evict_inplace: score -> pool -> select, then the kept rows move to the front of
-    every unit of K and V (written in place).  Returns {"idx", "scores", "lse"}."""
+    every unit of K and V (written in place; with ``paging``, to the first positions of every
+    sequence's pages).  Returns {"idx", "scores", "lse"}."""
     _check_cache(K, "K")
     _check_cache(V, "V")
     dev = K.device
@@ -210,17 +263,20 @@ def evict_inplace(p: Problem, K: torch.Tensor, V: torch.Tensor, Q: Optional[torc
     o.setdefault("lse", None)
     if ws is None:
         ws = workspace(p, dev)
-    bufs = B.dge_buffers(K=B.tensor_desc(K), V=B.tensor_desc(V), Q=B.tensor_desc(Q),
+    pg, pg_ptr = _paging_ptr(paging, K)
+    bufs = B.dge_buffers(K=_kv_desc(K, paging), V=_kv_desc(V, paging), Q=B.tensor_desc(Q),
                          scores=B.ptr(o["scores"]), idx=B.ptr(o["idx"]),
                          lse_in=_lse_arg(p, lse_in),
-                         lse_out=B.ptr(o["lse"]) if want_lse and lse_in is None else 0)
+                         lse_out=B.ptr(o["lse"]) if want_lse and lse_in is None else 0,
+                         paging=pg_ptr)
     B.dge_evict_inplace(p.c(), bufs, ws.data_ptr(), ws.numel(), _stream(stream))
     return o
 
 
 def diagnostics(p: Problem, Q: torch.Tensor, evicted: dict, lse: torch.Tensor, *, ws=None,
                 heldout_q: Optional[torch.Tensor] = None, K: Optional[torch.Tensor] = None,
-                V: Optional[torch.Tensor] = None, stream=None) -> dict:
+                V: Optional[torch.Tensor] = None, paging: Optional[Paging] = None,
+                stream=None) -> dict:
     """dge_diagnostics: per-row evicted mass (Problem.lse_shape), and per unit the
     attention-matching loss and the mean run of retained positions, for an eviction whose
     outputs (``evicted["Kc"]``, ``evicted["idx"]``) came from evict(); ``lse`` = the rows'
@@ -250,8 +306,10 @@ def diagnostics(p: Problem, Q: torch.Tensor, evicted: dict, lse: torch.Tensor, *
         out.heldout_mass = res["heldout_mass"].data_ptr()
         out.heldout_err = res["heldout_err"].data_ptr()
         out.heldout_gap = res["heldout_gap"].data_ptr()
-        bufs.K = B.tensor_desc(K)
-        bufs.V = B.tensor_desc(V)
+        bufs.K = _kv_desc(K, paging)
+        bufs.V = _kv_desc(V, paging)
+        if paging is not None:
+            pg, bufs.paging = _paging_ptr(paging, K)
     B.dge_diagnostics(p.c(), bufs, out, ws.data_ptr(), ws.numel(), _stream(stream))
     return res
 

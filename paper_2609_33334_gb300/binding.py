@@ -38,10 +38,15 @@ class dge_tensor(ctypes.Structure):
                 ("stride_head", c_int64), ("stride_pos", c_int64)]
 
 
+class dge_paging(ctypes.Structure):
+    _fields_ = [("block_table", c_void_p), ("page_size", c_int32), ("pages_per_seq", c_int32),
+                ("num_pages", c_int32), ("reserved", c_int32), ("stride_page", c_int64)]
+
+
 class dge_buffers(ctypes.Structure):
     _fields_ = [("K", dge_tensor), ("V", dge_tensor), ("Q", dge_tensor), ("scores", c_void_p),
                 ("idx", c_void_p), ("Kc", c_void_p), ("Vc", c_void_p), ("lse_in", c_void_p),
-                ("lse_out", c_void_p)]
+                ("lse_out", c_void_p), ("paging", POINTER(dge_paging))]
 
 
 class dge_diag(ctypes.Structure):
@@ -69,6 +74,7 @@ _LIB = None
 _P = POINTER(dge_problem)
 _B = POINTER(dge_buffers)
 _T = POINTER(dge_tensor)
+_G = POINTER(dge_paging)
 _SIGS = {
     "dge_workspace_size": [_P, POINTER(c_size_t)],
     "dge_packed_rows": [_P, POINTER(c_int64)],
@@ -80,6 +86,8 @@ _SIGS = {
     "dge_evict_inplace": [_P, _B, c_void_p, c_size_t, c_void_p],
     "dge_diagnostics": [_P, _B, ctypes.POINTER(dge_diag), c_void_p, c_size_t, c_void_p],
     "dge_compact_inplace": [_P, c_void_p, _T, _T, c_void_p, c_void_p],
+    "dge_compact_paged": [_P, _G, c_void_p, _T, _T, c_void_p, c_void_p, c_void_p, c_void_p],
+    "dge_compact_inplace_paged": [_P, _G, c_void_p, _T, _T, c_void_p, c_void_p],
     "dge_pyramid_budgets": [c_int32, c_int32, c_int32, POINTER(c_int32)],
     "dge_get_device_status": [c_void_p, c_void_p],
     "dge_status_string": [c_int],
@@ -169,6 +177,20 @@ def dge_compact_inplace(p: dge_problem, idx: int, K: dge_tensor, V: dge_tensor, 
     _check("dge_compact_inplace", _lib().dge_compact_inplace(ctypes.byref(p), idx,
                                                              ctypes.byref(K), ctypes.byref(V),
                                                              ws, stream))
+
+
+def dge_compact_paged(p: dge_problem, paging: dge_paging, idx: int, K: dge_tensor,
+                      V: dge_tensor, Kc: int, Vc: int, ws: int, stream: int) -> None:
+    _check("dge_compact_paged", _lib().dge_compact_paged(ctypes.byref(p), ctypes.byref(paging),
+                                                         idx, ctypes.byref(K), ctypes.byref(V),
+                                                         Kc, Vc, ws, stream))
+
+
+def dge_compact_inplace_paged(p: dge_problem, paging: dge_paging, idx: int, K: dge_tensor,
+                              V: dge_tensor, ws: int, stream: int) -> None:
+    _check("dge_compact_inplace_paged",
+           _lib().dge_compact_inplace_paged(ctypes.byref(p), ctypes.byref(paging), idx,
+                                            ctypes.byref(K), ctypes.byref(V), ws, stream))
 
 
 def dge_evict(p: dge_problem, bufs: dge_buffers, ws: int, ws_bytes: int, stream: int) -> None:

@@ -24,10 +24,15 @@ struct LayerTable {
     int64_t row_base[kMaxLayers];
 };
 
-// A bf16 tensor [layer][batch][head][pos][d] with element strides.
+// A bf16 tensor [layer][batch][head][pos][d] with element strides, or a paged cache: each
+// layer's pool of pages [page][slot][head][d] (s_page, s_pos = between slots, s_head), with
+// position p of sequence b in slot p % page_size of page bt[b * pps + p / page_size].
 struct TensorDesc {
     const __nv_bfloat16 *data;
     int64_t s_layer, s_batch, s_head, s_pos;
+    const int32_t *bt = nullptr;   // block table [b][pps] (paged caches only)
+    int page_size = 0, pps = 0, num_pages = 0;
+    int64_t s_page = 0;
 };
 
 // Everything a kernel needs to know about one eviction problem.
@@ -73,6 +78,25 @@ __device__ inline const __nv_bfloat16 *q_row_ptr(const TensorDesc &Q, const Geom
 __device__ inline const __nv_bfloat16 *kv_unit_ptr(const TensorDesc &T, int l, int bb, int h)
 {
     return T.data + l * T.s_layer + bb * T.s_batch + (int64_t)h * T.s_head;
+}
+
+// Page of position `pos` of sequence bb in a paged cache; page 0 for a table entry outside
+// the pool (the caller validated the table on the host side only when it was host-visible,
+// so a bad device entry is clamped rather than followed).
+__device__ inline int kv_page(const TensorDesc &T, int bb, int pos)
+{
+    const int page = __ldg(T.bt + (int64_t)bb * T.pps + pos / T.page_size);
+    return (page >= 0 && page < T.num_pages) ? page : 0;
+}
+
+// Row `pos` of unit (l, bb, h) of K or V, contiguous or paged.
+__device__ inline const __nv_bfloat16 *kv_row_ptr(const TensorDesc &T, int l, int bb, int h,
+                                                  int pos)
+{
+    if (T.bt)
+        return T.data + l * T.s_layer + (int64_t)kv_page(T, bb, pos) * T.s_page +
+               (int64_t)(pos % T.page_size) * T.s_pos + (int64_t)h * T.s_head;
+    return kv_unit_ptr(T, l, bb, h) + (int64_t)pos * T.s_pos;
 }
 
 // ---------------------------------------------------------------------------

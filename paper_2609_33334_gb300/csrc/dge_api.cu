@@ -289,6 +289,39 @@ TensorDesc desc(const dge_tensor &t)
     return d;
 }
 
+// A paged cache's geometry (NULL: contiguous).  page_size: 16, 32, 64 or a multiple of 128,
+// so a 128-key tile spans at most 8 pages and every TMA box starts 1024-byte aligned.
+int check_paging(const dge_paging *pg, int64_t n)
+{
+    if (!pg)
+        return DGE_OK;
+    if (!pg->block_table || pg->num_pages < 1 || pg->stride_page <= 0 || pg->reserved != 0)
+        return DGE_ERR_INVALID_ARG;
+    const int ps = pg->page_size;
+    if (!(ps == 16 || ps == 32 || ps == 64 || (ps >= 128 && ps % 128 == 0)))
+        return DGE_ERR_UNSUPPORTED;
+    if ((int64_t)pg->pages_per_seq * ps < n)
+        return DGE_ERR_INVALID_ARG;
+    if (((uintptr_t)pg->block_table & 3) || (pg->stride_page & 7))
+        return DGE_ERR_UNSUPPORTED;
+    return DGE_OK;
+}
+
+// K or V, contiguous or paged.
+TensorDesc kv_desc(const dge_tensor &t, const dge_paging *pg)
+{
+    TensorDesc d = desc(t);
+    if (pg) {
+        d.bt = pg->block_table;
+        d.page_size = pg->page_size;
+        d.pps = pg->pages_per_seq;
+        d.num_pages = pg->num_pages;
+        d.s_page = pg->stride_page;
+        d.s_batch = 0;
+    }
+    return d;
+}
+
 int check_ws(const Plan &plan, void *ws, size_t ws_bytes)
 {
     if (!ws)
@@ -529,14 +562,15 @@ int dge_score(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
     if (plan.g.variant == DGE_VARIANT_STREAMING || !bufs || !bufs->scores)
         return DGE_ERR_INVALID_ARG;
     if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->Q)) != DGE_OK ||
+        (rc = check_paging(bufs->paging, plan.g.n)) != DGE_OK ||
         (rc = check_ws(plan, ws, ws_bytes)) != DGE_OK)
         return rc;
     if (((uintptr_t)bufs->scores & 3) != 0 || !lse_ptrs_ok(bufs))
         return DGE_ERR_UNSUPPORTED;
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
     DGE_CHECK_CUDA(cudaMemsetAsync(ws, 0, sizeof(uint32_t), stream), "status clear");
-    if ((rc = run_scoring(plan, desc(bufs->K), desc(bufs->Q), ws, stream, bufs->lse_in,
-                          bufs->lse_out)) != DGE_OK)
+    if ((rc = run_scoring(plan, kv_desc(bufs->K, bufs->paging), desc(bufs->Q), ws, stream,
+                          bufs->lse_in, bufs->lse_out)) != DGE_OK)
         return rc;
     DGE_LAUNCH("pool", stream, launch_pool(ws_at<float>(ws, plan.off_raw), bufs->scores, plan.g.U, plan.g.P,
                                plan.g.pool, plan.g.pool_kernel, stream));
@@ -566,8 +600,9 @@ int dge_select(const dge_problem *p, const float *scores, int32_t *idx, void *st
     return DGE_OK;
 }
 
-int dge_compact(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
-                const dge_tensor *V, void *Kc, void *Vc, void *ws, void *stream_)
+int dge_compact_paged(const dge_problem *p, const dge_paging *paging, const int32_t *idx,
+                      const dge_tensor *K, const dge_tensor *V, void *Kc, void *Vc, void *ws,
+                      void *stream_)
 {
     Plan plan;
     int rc = make_plan(p, plan);
@@ -575,15 +610,24 @@ int dge_compact(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
         return rc;
     if (!idx || !K || !V || !Kc || !Vc)
         return DGE_ERR_INVALID_ARG;
-    if ((rc = check_tensor(*K)) != DGE_OK || (rc = check_tensor(*V)) != DGE_OK)
+    if ((rc = check_tensor(*K)) != DGE_OK || (rc = check_tensor(*V)) != DGE_OK ||
+        (rc = check_paging(paging, plan.g.n)) != DGE_OK)
         return rc;
     if (((uintptr_t)Kc & 15) || ((uintptr_t)Vc & 15) || ((uintptr_t)idx & 3) ||
         ((uintptr_t)ws & 255))
         return DGE_ERR_UNSUPPORTED;
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
-    DGE_LAUNCH("compact", stream, launch_compact(plan.g, plan.layers, idx, nullptr, desc(*K), desc(*V), Kc, Vc,
-                                  false, static_cast<uint32_t *>(ws), stream));
+    DGE_LAUNCH("compact", stream,
+               launch_compact(plan.g, plan.layers, idx, nullptr, kv_desc(*K, paging),
+                              kv_desc(*V, paging), Kc, Vc, false, static_cast<uint32_t *>(ws),
+                              stream));
     return DGE_OK;
+}
+
+int dge_compact(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
+                const dge_tensor *V, void *Kc, void *Vc, void *ws, void *stream)
+{
+    return dge_compact_paged(p, nullptr, idx, K, V, Kc, Vc, ws, stream);
 }
 
 }  // extern "C"
@@ -601,14 +645,15 @@ int evict_impl(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t w
         return rc;
     if (!bufs || !bufs->idx || (!inplace && (!bufs->Kc || !bufs->Vc)))
         return DGE_ERR_INVALID_ARG;
-    if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK)
+    if ((rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK ||
+        (rc = check_paging(bufs->paging, plan.g.n)) != DGE_OK)
         return rc;
     if ((!inplace && (((uintptr_t)bufs->Kc & 15) || ((uintptr_t)bufs->Vc & 15))) ||
         ((uintptr_t)bufs->idx & 3) || ((uintptr_t)bufs->scores & 3) || !lse_ptrs_ok(bufs))
         return DGE_ERR_UNSUPPORTED;
     const Geometry &g = plan.g;
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
-    const TensorDesc K = desc(bufs->K), V = desc(bufs->V);
+    const TensorDesc K = kv_desc(bufs->K, bufs->paging), V = kv_desc(bufs->V, bufs->paging);
     uint32_t *status = static_cast<uint32_t *>(ws);
     if (g.variant == DGE_VARIANT_STREAMING) {
         if (ws && ((uintptr_t)ws & 255))
@@ -703,7 +748,8 @@ int dge_diagnostics(const dge_problem *p, const dge_buffers *bufs, const dge_dia
         if (!out->heldout_mass || !out->heldout_err || !out->heldout_gap)
             return DGE_ERR_INVALID_ARG;
         if ((rc = check_tensor(out->heldout_q)) != DGE_OK ||
-            (rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK)
+            (rc = check_tensor(bufs->K)) != DGE_OK || (rc = check_tensor(bufs->V)) != DGE_OK ||
+            (rc = check_paging(bufs->paging, g.n)) != DGE_OK)
             return rc;
         if (((uintptr_t)out->heldout_mass & 3) || ((uintptr_t)out->heldout_err & 3) ||
             ((uintptr_t)out->heldout_gap & 3) || !heldout_supported(g))
@@ -746,14 +792,15 @@ int dge_diagnostics(const dge_problem *p, const dge_buffers *bufs, const dge_dia
                            out->l_match, out->run_length, stream));
     if (out->heldout_q.data)
         DGE_LAUNCH("heldout", stream,
-                   launch_heldout(desc(out->heldout_q), desc(bufs->K), desc(bufs->V), bufs->idx,
+                   launch_heldout(desc(out->heldout_q), kv_desc(bufs->K, bufs->paging),
+                                  kv_desc(bufs->V, bufs->paging), bufs->idx,
                                   g, plan.layers, out->heldout_mass, out->heldout_err,
                                   out->heldout_gap, stream));
     return DGE_OK;
 }
 
-int dge_compact_inplace(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
-                        const dge_tensor *V, void *ws, void *stream_)
+int dge_compact_inplace_paged(const dge_problem *p, const dge_paging *paging, const int32_t *idx,
+                              const dge_tensor *K, const dge_tensor *V, void *ws, void *stream_)
 {
     Plan plan;
     int rc = make_plan(p, plan);
@@ -761,15 +808,23 @@ int dge_compact_inplace(const dge_problem *p, const int32_t *idx, const dge_tens
         return rc;
     if (!idx || !K || !V)
         return DGE_ERR_INVALID_ARG;
-    if ((rc = check_tensor(*K)) != DGE_OK || (rc = check_tensor(*V)) != DGE_OK)
+    if ((rc = check_tensor(*K)) != DGE_OK || (rc = check_tensor(*V)) != DGE_OK ||
+        (rc = check_paging(paging, plan.g.n)) != DGE_OK)
         return rc;
     if (((uintptr_t)idx & 3) || ((uintptr_t)ws & 255))
         return DGE_ERR_UNSUPPORTED;
     cudaStream_t stream = static_cast<cudaStream_t>(stream_);
     DGE_LAUNCH("compact_inplace", stream,
-               launch_compact_inplace(plan.g, plan.layers, idx, nullptr, desc(*K), desc(*V),
-                                      false, static_cast<uint32_t *>(ws), stream));
+               launch_compact_inplace(plan.g, plan.layers, idx, nullptr, kv_desc(*K, paging),
+                                      kv_desc(*V, paging), false, static_cast<uint32_t *>(ws),
+                                      stream));
     return DGE_OK;
+}
+
+int dge_compact_inplace(const dge_problem *p, const int32_t *idx, const dge_tensor *K,
+                        const dge_tensor *V, void *ws, void *stream)
+{
+    return dge_compact_inplace_paged(p, nullptr, idx, K, V, ws, stream);
 }
 
 int dge_pyramid_budgets(int32_t B, int32_t w, int32_t L, int32_t *out)

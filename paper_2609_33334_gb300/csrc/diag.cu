@@ -125,14 +125,12 @@ heldout_kernel(TensorDesc Qh, TensorDesc K, TensorDesc V, const int32_t *__restr
 #pragma unroll
     for (int e = 0; e < E; ++e)
         qv[e] = __bfloat162float(q[lane * E + e]) * g.scale_log2;
-    const __nv_bfloat16 *Ku = K.data + l * K.s_layer + bb * K.s_batch + h * K.s_head;
-    const __nv_bfloat16 *Vu = V.data + l * V.s_layer + bb * V.s_batch + h * V.s_head;
     float mx = -INFINITY, z[2] = {0.f, 0.f}, o[2][E];
 #pragma unroll
     for (int e = 0; e < E; ++e)
         o[0][e] = o[1][e] = 0.f;
     for (int j = warp; j < n; j += kHoWarps) {
-        const __nv_bfloat16 *kr = Ku + (int64_t)j * K.s_pos + lane * E;
+        const __nv_bfloat16 *kr = kv_row_ptr(K, l, bb, h, j) + lane * E;
         float s = 0.f;
 #pragma unroll
         for (int e = 0; e < E; ++e)
@@ -154,7 +152,7 @@ heldout_kernel(TensorDesc Qh, TensorDesc K, TensorDesc V, const int32_t *__restr
         const float w = ex2(s - mx);
         const int set = (keep_bits[j >> 5] >> (j & 31)) & 1u ? 0 : 1;   // 0 kept, 1 evicted
         z[set] += w;
-        const __nv_bfloat16 *vr = Vu + (int64_t)j * V.s_pos + lane * E;
+        const __nv_bfloat16 *vr = kv_row_ptr(V, l, bb, h, j) + lane * E;
 #pragma unroll
         for (int e = 0; e < E; ++e)
             o[set][e] = fmaf(w, __bfloat162float(vr[e]), o[set][e]);

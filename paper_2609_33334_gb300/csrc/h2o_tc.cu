@@ -73,6 +73,7 @@ static_assert(kNumBars * 8 + 16 + 16 * 4 <= kCtrlBytes, "control block");
 
 struct H2oArgs {
     Geometry g;
+    tc::KPaging kp;    // K through a block table (kp.bt != nullptr)
     int phase;         // 1: row normalisers, 2: column sums
     int pb;            // positions per query block
     int rows;          // G * pb
@@ -242,6 +243,7 @@ __device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
         }
 }
 
+template <bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
 h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
               const H2oArgs a)
@@ -342,14 +344,13 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                     ptx::mbar_arrive_expect_tx(&sm.bar[kBarStatFull + sb],
                                                a.phase == 1 ? qbytes : kbytes);
                     flag[kFlagStatArm + sb] = (int)sph;
-                    for (int s = 0; s < a.nslab; ++s) {
-                        if (a.phase == 1)
-                            ptx::tma_load_5d_hint(sdst + s * sslab, &tmQ, &sm.bar[kBarStatFull + sb],
-                                                  s * 64, T.blk * a.pb, h * g.G, bb, l, once_pol);
-                        else
-                            ptx::tma_load_5d_hint(sdst + s * sslab, &tmK, &sm.bar[kBarStatFull + sb],
-                                                  s * 64, T.blk * kTile, h, bb, l, once_pol);
+                    for (int s = 0; s < a.nslab && a.phase == 1; ++s) {
+                        ptx::tma_load_5d_hint(sdst + s * sslab, &tmQ, &sm.bar[kBarStatFull + sb],
+                                              s * 64, T.blk * a.pb, h * g.G, bb, l, once_pol);
                     }
+                    if (a.phase == 2)
+                        tc::load_k_tile<kPaged>(sdst, sslab, a.nslab, &tmK, &sm.bar[kBarStatFull + sb],
+                                        T.blk * kTile, l, bb, h, a.kp, once_pol);
                     if (++sb == 2) {
                         sb = 0;
                         sph ^= 1;
@@ -363,17 +364,15 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                         ptx::mbar_arrive_expect_tx(&sm.bar[kBarRingFull + rs],
                                                    a.phase == 1 ? kbytes : qbytes);
                         flag[kFlagRingArm + rs] = (int)rph;
-                        for (int s = 0; s < a.nslab; ++s) {
-                            if (a.phase == 1)
-                                ptx::tma_load_5d_hint(rdst + s * rslab, &tmK,
-                                                      &sm.bar[kBarRingFull + rs], s * 64, i * kTile,
-                                                      h, bb, l, shared_pol);
-                            else
+                        if (a.phase == 1)
+                            tc::load_k_tile<kPaged>(rdst, rslab, a.nslab, &tmK, &sm.bar[kBarRingFull + rs],
+                                            i * kTile, l, bb, h, a.kp, shared_pol);
+                        else
+                            for (int s = 0; s < a.nslab; ++s)
                                 ptx::tma_load_5d_hint(rdst + s * rslab, &tmQ,
                                                       &sm.bar[kBarRingFull + rs], s * 64,
                                                       (T.first + i) * a.pb, h * g.G, bb, l,
                                                       shared_pol);
-                        }
                         if (++rs == kStages) {
                             rs = 0;
                             rph ^= 1;
@@ -792,7 +791,7 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
                           uint32_t *status, cudaStream_t stream, bool *encoded)
 {
     CUtensorMap tmK, tmQ;
-    *encoded = tc::encode_5d(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d, kTile, 1) &&
+    *encoded = tc::encode_k_map(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d) &&
                tc::encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.n, g.d, plan.pb, g.G);
     if (!*encoded)
         return cudaSuccess;
@@ -805,6 +804,7 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
 
     H2oArgs a;
     a.g = g;
+    a.kp = tc::k_paging(K, g.n);
     a.phase = phase;
     a.pb = plan.pb;
     a.rows = plan.rows;
@@ -828,12 +828,12 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
     if (a.items == 0)
         return cudaSuccess;
     const size_t smem = plan.smem[phase - 1];
-    err = cudaFuncSetAttribute(h2o_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)smem);
+    auto kernel = K.bt ? h2o_tc_kernel<true> : h2o_tc_kernel<false>;
+    err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (err != cudaSuccess)
         return err;
     const int64_t grid = a.items < sms ? a.items : sms;
-    h2o_tc_kernel<<<(unsigned)grid, kThreads, smem, stream>>>(tmK, tmQ, a);
+    kernel<<<(unsigned)grid, kThreads, smem, stream>>>(tmK, tmQ, a);
     return cudaGetLastError();
 }
 

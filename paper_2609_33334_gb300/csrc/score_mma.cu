@@ -52,7 +52,7 @@ __device__ void stage_rows(__nv_bfloat16 *sQ, const TensorDesc &Q, const Geometr
 
 // Stage keys [k0, k0 + kTileKeys) of one unit, zero-filling keys >= k_lim.
 template <int D, int KEYS>
-__device__ void stage_keys(__nv_bfloat16 *sK, const __nv_bfloat16 *Ku, int64_t s_pos, int k0,
+__device__ void stage_keys(__nv_bfloat16 *sK, const TensorDesc &K, int l, int bb, int h, int k0,
                            int k_lim)
 {
     constexpr int V = D / 8;
@@ -61,7 +61,7 @@ __device__ void stage_keys(__nv_bfloat16 *sK, const __nv_bfloat16 *Ku, int64_t s
         const int key = k0 + r;
         __nv_bfloat16 *dst = sK + r * Pad<D>::kStride + c * 8;
         if (key < k_lim)
-            cp_async_16(dst, Ku + (int64_t)key * s_pos + c * 8, 16);
+            cp_async_16(dst, kv_row_ptr(K, l, bb, h, key) + c * 8, 16);
         else
             *reinterpret_cast<int4 *>(dst) = make_int4(0, 0, 0, 0);
     }
@@ -152,15 +152,14 @@ lse_partial_kernel(TensorDesc K, TensorDesc Q, Geometry g, int rows_per_block, i
     if (k_lo < k_hi) {
         __nv_bfloat16 *sQ = reinterpret_cast<__nv_bfloat16 *>(smem);
         __nv_bfloat16 *sK = sQ + rows_pad * Pad<D>::kStride;
-        const __nv_bfloat16 *Ku = kv_unit_ptr(K, l, bb, h);
         stage_rows<D>(sQ, Q, g, l, bb, h, r0, rows, rows_pad, rows_per_head);
-        stage_keys<D, kTileKeys>(sK, Ku, K.s_pos, k_lo, k_hi);
+        stage_keys<D, kTileKeys>(sK, K, l, bb, h, k_lo, k_hi);
         cp_async_commit();
         const int ntiles = (k_hi - k_lo + kTileKeys - 1) / kTileKeys;
         for (int t = 0; t < ntiles; ++t) {
             if (t + 1 < ntiles) {
-                stage_keys<D, kTileKeys>(sK + ((t + 1) & 1) * kTileKeys * Pad<D>::kStride, Ku,
-                                         K.s_pos, k_lo + (t + 1) * kTileKeys, k_hi);
+                stage_keys<D, kTileKeys>(sK + ((t + 1) & 1) * kTileKeys * Pad<D>::kStride, K, l,
+                                         bb, h, k_lo + (t + 1) * kTileKeys, k_hi);
                 cp_async_commit();
                 cp_async_wait<1>();
             } else {
@@ -283,15 +282,14 @@ colsum_rows_kernel(TensorDesc K, TensorDesc Q, Geometry g, int chunk_keys, int n
 
     __nv_bfloat16 *sQ = reinterpret_cast<__nv_bfloat16 *>(smem);
     __nv_bfloat16 *sK = sQ + rows_pad * Pad<D>::kStride;
-    const __nv_bfloat16 *Ku = kv_unit_ptr(K, l, bb, h);
     stage_rows<D>(sQ, Q, g, l, bb, h, 0, rows, rows_pad, g.m);
-    stage_keys<D, kTileKeys>(sK, Ku, K.s_pos, k_lo, k_hi);
+    stage_keys<D, kTileKeys>(sK, K, l, bb, h, k_lo, k_hi);
     cp_async_commit();
     const int ntiles = (k_hi - k_lo + kTileKeys - 1) / kTileKeys;
     for (int t = 0; t < ntiles; ++t) {
         if (t + 1 < ntiles) {
-            stage_keys<D, kTileKeys>(sK + ((t + 1) & 1) * kTileKeys * Pad<D>::kStride, Ku,
-                                     K.s_pos, k_lo + (t + 1) * kTileKeys, k_hi);
+            stage_keys<D, kTileKeys>(sK + ((t + 1) & 1) * kTileKeys * Pad<D>::kStride, K, l, bb,
+                                     h, k_lo + (t + 1) * kTileKeys, k_hi);
             cp_async_commit();
             cp_async_wait<1>();
         } else {
@@ -372,8 +370,7 @@ colsum_keys_kernel(TensorDesc K, TensorDesc Q, Geometry g, int nkb,
 
     __nv_bfloat16 *sK = reinterpret_cast<__nv_bfloat16 *>(smem);
     __nv_bfloat16 *sQ = sK + kKeyBlock * Pad<D>::kStride;  // [2][kRowTile][stride]
-    const __nv_bfloat16 *Ku = kv_unit_ptr(K, l, bb, h);
-    stage_keys<D, kKeyBlock>(sK, Ku, K.s_pos, k_lo, k_hi);
+    stage_keys<D, kKeyBlock>(sK, K, l, bb, h, k_lo, k_hi);
     cp_async_commit();
 
     // Row tiles: for every query head of the group, positions from the tile

@@ -70,6 +70,7 @@ constexpr int kFlagAbort = tc::kFlagAbort, kFlagKArm = 4, kFlagQArm = 8, kFlagSA
 
 struct TcArgs {
     Geometry g;
+    tc::KPaging kp;    // K through a block table (kp.bt != nullptr)
     int rows;          // stacked rows of a sub-unit: gsub heads x m (all of R when nrb == 1)
     int nrb, gsub;     // sub-units (row blocks) per unit, query heads per sub-unit
     int r_pad, r4, nslab, kstages;
@@ -315,7 +316,7 @@ __device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
 // clock reads cost nothing when tracing is off).  kFx: units split into row blocks whose
 // column sums meet in fixed point (a separate build, so the whole-unit path carries none of
 // it: its epilogue is latency-bound and slowed by 5% with it).
-template <bool kTr, bool kFx>
+template <bool kTr, bool kFx, bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
 score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
                 const TcArgs a)
@@ -437,10 +438,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         ptx::mbar_arrive_expect_tx(&sm.bar[kBarKFull + ks],
                                                    (uint32_t)a.nslab * kSlabBytes);
                         flag[kFlagKArm + ks] = (int)kph;
-                        for (int s = 0; s < a.nslab; ++s)
-                            ptx::tma_load_5d_hint(sm.k + ((size_t)ks * a.nslab + s) * kSlabBytes,
-                                                  &tmK, &sm.bar[kBarKFull + ks], s * 64,
-                                                  T.k_lo + tile * kTile, h, bb, l, pol);
+                        tc::load_k_tile<kPaged>(sm.k + (size_t)ks * a.nslab * kSlabBytes, kSlabBytes,
+                                        a.nslab, &tmK, &sm.bar[kBarKFull + ks],
+                                        T.k_lo + tile * kTile, l, bb, h, a.kp, pol);
                         if (++ks == a.kstages) {
                             ks = 0;
                             kph ^= 1;
@@ -1021,6 +1021,43 @@ bool have_tensor_maps()
     return encode_fn_impl() != nullptr;
 }
 
+bool encode_k_map(CUtensorMap *map, const TensorDesc &t, int L, int b, int Hkv, int n, int d)
+{
+    if (!t.bt)
+        return encode_5d(map, t, L, b, Hkv, n, d, 128, 1);
+    Encode fn = encode_fn_impl();
+    if (!fn)
+        return false;
+    // [L][page][slot][head][d]: boxes of one head, min(page_size, 128) slots.  A pool of one
+    // layer may carry any layer stride; give the map a nonzero one.
+    const int64_t s_layer = t.s_layer != 0 ? t.s_layer : t.s_page * t.num_pages;
+    const cuuint64_t dims[5] = {(cuuint64_t)d, (cuuint64_t)Hkv, (cuuint64_t)t.page_size,
+                                (cuuint64_t)t.num_pages, (cuuint64_t)L};
+    const cuuint64_t strides[4] = {(cuuint64_t)t.s_head * 2, (cuuint64_t)t.s_pos * 2,
+                                   (cuuint64_t)t.s_page * 2, (cuuint64_t)s_layer * 2};
+    const cuuint32_t box[5] = {64, 1, (cuuint32_t)(t.page_size < 128 ? t.page_size : 128), 1, 1};
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    for (int i = 0; i < 4; ++i)
+        if (strides[i] == 0 || strides[i] % 16 != 0)
+            return false;
+    (void)b;
+    (void)n;
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<__nv_bfloat16 *>(t.data), dims,
+              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+KPaging k_paging(const TensorDesc &t, int n)
+{
+    KPaging p;
+    p.bt = t.bt;
+    p.page_size = t.page_size;
+    p.pps = t.pps;
+    p.num_pages = t.num_pages;
+    p.n = n;
+    return p;
+}
+
 }  // namespace tc
 
 void tc_set_trace(unsigned long long *buffer, int cta)
@@ -1099,7 +1136,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
                             bool *encoded)
 {
     CUtensorMap tmK, tmQ;
-    *encoded = tc::encode_5d(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d, kTile, 1) &&
+    *encoded = tc::encode_k_map(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d) &&
                tc::encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.m, g.d, g.m, plan.gsub);
     if (!*encoded)
         return cudaSuccess;
@@ -1112,6 +1149,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
 
     TcArgs a;
     a.g = g;
+    a.kp = tc::k_paging(K, g.n);
     a.rows = plan.rows;
     a.nrb = plan.nrb;
     a.gsub = plan.gsub;
@@ -1149,10 +1187,14 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.trace = g_trace;
     a.trace_cta = g_trace_cta;
 
-    // The traced build covers whole units only; row blocks run untraced.
+    // The traced build covers whole, contiguous units only; row blocks and paged caches run
+    // untraced.
     void (*kernel)(const CUtensorMap, const CUtensorMap, const TcArgs) =
-        plan.nrb > 1 ? score_tc_kernel<false, true>
-                     : (a.trace ? score_tc_kernel<true, false> : score_tc_kernel<false, false>);
+        K.bt ? (plan.nrb > 1 ? score_tc_kernel<false, true, true>
+                             : score_tc_kernel<false, false, true>)
+             : (plan.nrb > 1 ? score_tc_kernel<false, true, false>
+                             : (a.trace ? score_tc_kernel<true, false, false>
+                                        : score_tc_kernel<false, false, false>));
     err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                (int)plan.smem);
     if (err != cudaSuccess)

@@ -619,7 +619,18 @@ cudaError_t launch_streaming_indices(const Geometry &g, const LayerTable &layers
 // computed in place (and written to idx).
 constexpr int kGatherRows = 64;
 
-template <int D>
+// Row `pos` of a unit: contiguous (from the unit's base) or through the block table.
+template <bool kPaged>
+__device__ __forceinline__ const __nv_bfloat16 *gather_row(const TensorDesc &T,
+                                                           const __nv_bfloat16 *unit, int l,
+                                                           int bb, int h, int pos)
+{
+    if constexpr (kPaged)
+        return kv_row_ptr(T, l, bb, h, pos);
+    return unit + (int64_t)pos * T.s_pos;
+}
+
+template <int D, bool kPaged>
 __global__ void __launch_bounds__(256)
 compact_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__ idx_out, TensorDesc K,
                TensorDesc V, __nv_bfloat16 *__restrict__ Kc, __nv_bfloat16 *__restrict__ Vc,
@@ -652,8 +663,10 @@ compact_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__ idx_out
                 set_status(status, DGE_ERR_INVALID_ARG);
             continue;
         }
-        const int4 kv = *reinterpret_cast<const int4 *>(Ku + (int64_t)pos * K.s_pos + part * 8);
-        const int4 vv = *reinterpret_cast<const int4 *>(Vu + (int64_t)pos * V.s_pos + part * 8);
+        const int4 kv = *reinterpret_cast<const int4 *>(
+            gather_row<kPaged>(K, Ku, l, bb, h, pos) + part * 8);
+        const int4 vv = *reinterpret_cast<const int4 *>(
+            gather_row<kPaged>(V, Vu, l, bb, h, pos) + part * 8);
         *reinterpret_cast<int4 *>(Kc + (base + r) * D + part * 8) = kv;
         *reinterpret_cast<int4 *>(Vc + (base + r) * D + part * 8) = vv;
     }
@@ -666,7 +679,9 @@ compact_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__ idx_out
 // registers before the block barrier and written after it, so a row that is both read and
 // written within the chunk is read first; rows written by earlier chunks lie below every
 // later source row.  A position outside [r, n) is reported (DGE_ERR_INVALID_ARG) and skipped.
-template <int D>
+// A paged cache keeps the same order on the sequence's positions: row r of the unit goes to
+// position r through the block table.
+template <int D, bool kPaged>
 __global__ void __launch_bounds__(256)
 compact_inplace_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__ idx_out,
                        TensorDesc K, TensorDesc V, SelectParams p, int implicit, uint32_t *status)
@@ -702,8 +717,10 @@ compact_inplace_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__
                     if (part == 0)
                         set_status(status, DGE_ERR_INVALID_ARG);
                 } else if (pos != r) {
-                    kv[i] = *reinterpret_cast<const int4 *>(Ku + (int64_t)pos * K.s_pos + part * 8);
-                    vv[i] = *reinterpret_cast<const int4 *>(Vu + (int64_t)pos * V.s_pos + part * 8);
+                    kv[i] = *reinterpret_cast<const int4 *>(
+                        gather_row<kPaged>(K, Ku, l, bb, h, pos) + part * 8);
+                    vv[i] = *reinterpret_cast<const int4 *>(
+                        gather_row<kPaged>(V, Vu, l, bb, h, pos) + part * 8);
                     dst[i] = r;
                 }
             }
@@ -712,8 +729,12 @@ compact_inplace_kernel(const int32_t *__restrict__ idx_in, int32_t *__restrict__
 #pragma unroll
         for (int i = 0; i < kPasses; ++i)
             if (dst[i] >= 0) {
-                *reinterpret_cast<int4 *>(Ku + (int64_t)dst[i] * K.s_pos + part * 8) = kv[i];
-                *reinterpret_cast<int4 *>(Vu + (int64_t)dst[i] * V.s_pos + part * 8) = vv[i];
+                *reinterpret_cast<int4 *>(
+                    const_cast<__nv_bfloat16 *>(gather_row<kPaged>(K, Ku, l, bb, h, dst[i])) +
+                    part * 8) = kv[i];
+                *reinterpret_cast<int4 *>(
+                    const_cast<__nv_bfloat16 *>(gather_row<kPaged>(V, Vu, l, bb, h, dst[i])) +
+                    part * 8) = vv[i];
             }
     }
 }
@@ -728,12 +749,11 @@ cudaError_t launch_compact_inplace(const Geometry &g, const LayerTable &layers,
     p.layers = layers;
     if (g.U == 0)
         return cudaSuccess;
-    if (g.d == 128)
-        compact_inplace_kernel<128><<<(unsigned)g.U, 256, 0, stream>>>(
-            idx_in, idx_out, K, V, p, implicit ? 1 : 0, status);
-    else
-        compact_inplace_kernel<64><<<(unsigned)g.U, 256, 0, stream>>>(
-            idx_in, idx_out, K, V, p, implicit ? 1 : 0, status);
+    auto kernel = g.d == 128 ? (K.bt ? compact_inplace_kernel<128, true>
+                                     : compact_inplace_kernel<128, false>)
+                             : (K.bt ? compact_inplace_kernel<64, true>
+                                     : compact_inplace_kernel<64, false>);
+    kernel<<<(unsigned)g.U, 256, 0, stream>>>(idx_in, idx_out, K, V, p, implicit ? 1 : 0, status);
     return cudaGetLastError();
 }
 
@@ -751,14 +771,12 @@ cudaError_t launch_compact(const Geometry &g, const LayerTable &layers, const in
     if (nrb == 0)
         return cudaSuccess;
     const int64_t blocks = g.U * nrb;
-    if (g.d == 128)
-        compact_kernel<128><<<(unsigned)blocks, 256, 0, stream>>>(
-            idx_in, idx_out, K, V, static_cast<__nv_bfloat16 *>(Kc),
-            static_cast<__nv_bfloat16 *>(Vc), p, nrb, implicit ? 1 : 0, status);
-    else
-        compact_kernel<64><<<(unsigned)blocks, 256, 0, stream>>>(
-            idx_in, idx_out, K, V, static_cast<__nv_bfloat16 *>(Kc),
-            static_cast<__nv_bfloat16 *>(Vc), p, nrb, implicit ? 1 : 0, status);
+    auto kernel = g.d == 128 ? (K.bt ? compact_kernel<128, true> : compact_kernel<128, false>)
+                             : (K.bt ? compact_kernel<64, true> : compact_kernel<64, false>);
+    kernel<<<(unsigned)blocks, 256, 0, stream>>>(idx_in, idx_out, K, V,
+                                                 static_cast<__nv_bfloat16 *>(Kc),
+                                                 static_cast<__nv_bfloat16 *>(Vc), p, nrb,
+                                                 implicit ? 1 : 0, status);
     return cudaGetLastError();
 }
 

@@ -89,12 +89,64 @@ __device__ __forceinline__ void transpose_sum16(float (&a)[16], int lane)
     }
 }
 
+// K of a paged cache as the tcgen05 producers see it (bt == nullptr: contiguous).
+struct KPaging {
+    const int32_t *bt;   // block table [b][pps]
+    int page_size, pps, num_pages, n;
+};
+
+// Largest number of pages a 128-key tile spans (page sizes 16, 32, 64 or multiples of 128).
+constexpr int kMaxTilePages = 8;
+
+// One 128-key tile of K (nslab slabs of 64 columns, slab_bytes apart) into shared memory with
+// TMA, completing on `bar`: one box per slab from a contiguous cache (map over
+// [L][b][Hkv][n][d]), or one box of min(page_size, 128) slots per page from a paged one (map
+// over [L][page][slot][Hkv][d]).  Page ids are all read before the first copy is issued (one
+// round trip a tile); positions past the cache read page 0, whose rows the callers mask.
+template <bool kPaged>
+__device__ __forceinline__ void load_k_tile(uint8_t *dst, uint32_t slab_bytes, int nslab,
+                                            const CUtensorMap *map, uint64_t *bar, int k0, int l,
+                                            int bb, int h, const KPaging &pg, uint64_t policy)
+{
+    if constexpr (!kPaged) {
+        for (int s = 0; s < nslab; ++s)
+            ptx::tma_load_5d_hint(dst + s * slab_bytes, map, bar, s * 64, k0, h, bb, l, policy);
+        return;
+    }
+    else {
+        const int rows = pg.page_size < 128 ? pg.page_size : 128;
+        const int npg = 128 / rows;
+        int page[kMaxTilePages];
+#pragma unroll
+        for (int j = 0; j < kMaxTilePages; ++j) {
+            const int pos = k0 + j * rows;
+            page[j] = 0;
+            if (j < npg && pos < pg.n) {
+                const int pid = __ldg(pg.bt + (int64_t)bb * pg.pps + pos / pg.page_size);
+                page[j] = (pid >= 0 && pid < pg.num_pages) ? pid : 0;
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < kMaxTilePages; ++j)
+            if (j < npg) {
+                const int pos = k0 + j * rows;
+                const int slot = pos < pg.n ? pos % pg.page_size : 0;
+                for (int s = 0; s < nslab; ++s)
+                    ptx::tma_load_5d_hint(dst + s * slab_bytes + j * rows * 128, map, bar, s * 64,
+                                          h, slot, page[j], l, policy);
+            }
+    }
+}
+
 // Host: a 5-D TMA map over [L][b][heads][rows][d] (bf16, 128-byte swizzle) with box
 // {64, box_rows, box_heads, 1, 1}; false when the driver entry point is missing or the strides
 // are not 16-byte multiples.
 bool encode_5d(CUtensorMap *map, const TensorDesc &t, int L, int b, int heads, int rows, int d,
                int box_rows, int box_heads);
 bool have_tensor_maps();
+// Host: the K map of load_k_tile -- contiguous, or over a paged cache's pools (t.bt set).
+bool encode_k_map(CUtensorMap *map, const TensorDesc &t, int L, int b, int Hkv, int n, int d);
+KPaging k_paging(const TensorDesc &t, int n);
 
 }  // namespace tc
 }  // namespace dge

@@ -207,3 +207,44 @@ def _plant_spans(wl: Workload, seq: int, q: torch.Tensor, k: torch.Tensor, g) ->
 def bf16_bits(t: torch.Tensor) -> np.ndarray:
     """Raw bf16 bit patterns of a (CPU or CUDA) tensor as a contiguous uint16 array."""
     return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def paged_layout(cache: torch.Tensor, page_size: int, seed: int = 0, spare_pages: int = 3,
+                 extra_table_pages: int = 1) -> tuple:
+    """Lay a contiguous cache [L][b][Hkv][n][d] out as a paged one, the way a paged-attention
+    server keeps it: returns (pool [L][num_pages][page_size][Hkv][d], block_table int32
+    [b][pages_per_seq]).  Sequences get pages in a seeded random order (shared by all
+    layers), the pool has ``spare_pages`` pages no sequence uses, and the table has
+    ``extra_table_pages`` entries per sequence past the cache (set to -1).  Every slot that
+    holds no cache position is NaN, so a read of one shows in the results.  Pure layout: no
+    arithmetic of the method."""
+    L, b, Hkv, n, d = cache.shape
+    used = (n + page_size - 1) // page_size
+    pps = used + extra_table_pages
+    num_pages = b * used + spare_pages
+    rng = np.random.default_rng(seed)
+    perm = rng.permutation(num_pages)[:b * used].reshape(b, used)
+    table = np.full((b, pps), -1, dtype=np.int32)
+    table[:, :used] = perm
+    pool = torch.full((L, num_pages, page_size, Hkv, d), float("nan"), dtype=cache.dtype,
+                      device=cache.device)
+    for s in range(b):
+        for j in range(used):
+            lo, hi = j * page_size, min((j + 1) * page_size, n)
+            # [L][Hkv][rows][d] -> [L][rows][Hkv][d]
+            pool[:, int(perm[s, j]), :hi - lo] = cache[:, s, :, lo:hi].permute(0, 2, 1, 3)
+    return pool, torch.from_numpy(table).to(cache.device)
+
+
+def unpaged(pool: torch.Tensor, block_table: torch.Tensor, n: int) -> torch.Tensor:
+    """The contiguous cache [L][b][Hkv][n][d] that a paged one holds (inverse of paged_layout
+    on positions [0, n))."""
+    L, _, page_size, Hkv, d = pool.shape
+    b = block_table.shape[0]
+    out = torch.empty((L, b, Hkv, n, d), dtype=pool.dtype, device=pool.device)
+    table = block_table.cpu().numpy()
+    for s in range(b):
+        for j in range((n + page_size - 1) // page_size):
+            lo, hi = j * page_size, min((j + 1) * page_size, n)
+            out[:, s, :, lo:hi] = pool[:, int(table[s, j]), :hi - lo].permute(0, 2, 1, 3)
+    return out

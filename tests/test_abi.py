@@ -49,9 +49,12 @@ def test_struct_layout_matches_c():
     assert B.dge_problem.select_block.offset == 56
     assert B.dge_problem.budgets.offset == 64
     assert ctypes.sizeof(B.dge_tensor) == 40
-    assert ctypes.sizeof(B.dge_buffers) == 3 * 40 + 6 * 8
+    assert ctypes.sizeof(B.dge_buffers) == 3 * 40 + 7 * 8
     assert B.dge_buffers.lse_in.offset == 3 * 40 + 4 * 8
     assert B.dge_buffers.lse_out.offset == 3 * 40 + 5 * 8
+    assert B.dge_buffers.paging.offset == 3 * 40 + 6 * 8
+    assert ctypes.sizeof(B.dge_paging) == 32
+    assert B.dge_paging.stride_page.offset == 24
 
 
 def test_pyramid_budgets_paper_examples(lib):
@@ -177,3 +180,39 @@ def test_null_and_misaligned_arguments_rejected_before_launch(lib):
                                    None) == B.DGE_ERR_INVALID_ARG
     assert lib.dge_compact_inplace(ctypes.byref(p), 0x2002, ctypes.byref(t), ctypes.byref(t),
                                    None, None) == B.DGE_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(block_table=0), B.DGE_ERR_INVALID_ARG),
+    (dict(page_size=8), B.DGE_ERR_UNSUPPORTED),            # a 128-key tile would span 16 pages
+    (dict(page_size=48), B.DGE_ERR_UNSUPPORTED),
+    (dict(page_size=192), B.DGE_ERR_UNSUPPORTED),
+    (dict(pages_per_seq=63), B.DGE_ERR_INVALID_ARG),       # 63 * 16 < n = 1024
+    (dict(num_pages=0), B.DGE_ERR_INVALID_ARG),
+    (dict(reserved=1), B.DGE_ERR_INVALID_ARG),
+    (dict(stride_page=0), B.DGE_ERR_INVALID_ARG),
+    (dict(stride_page=12), B.DGE_ERR_UNSUPPORTED),
+    (dict(block_table=0x7002), B.DGE_ERR_UNSUPPORTED),     # misaligned table
+])
+def test_paging_validation(lib, kw, code):
+    """Bad paged-cache geometry is rejected before anything is enqueued, by every call that
+    takes K / V."""
+    p = _problem()
+    base = dict(block_table=0x7000, page_size=16, pages_per_seq=64, num_pages=200,
+                reserved=0, stride_page=16 * 2 * 64)
+    base.update(kw)
+    pg = B.dge_paging(**base)
+    t = B.dge_tensor(data=0x1000, stride_layer=200 * 16 * 2 * 64, stride_batch=0,
+                     stride_head=64, stride_pos=2 * 64)
+    bufs = B.dge_buffers(K=t, V=t, Q=t, scores=0x5000, idx=0x2000, Kc=0x3000, Vc=0x4000,
+                         paging=ctypes.pointer(pg))
+    need = ctypes.c_size_t(0)
+    assert lib.dge_workspace_size(ctypes.byref(p), ctypes.byref(need)) == 0
+    assert lib.dge_evict(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value, None) == code
+    assert lib.dge_evict_inplace(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value,
+                                 None) == code
+    assert lib.dge_score(ctypes.byref(p), ctypes.byref(bufs), 0x10000, need.value, None) == code
+    assert lib.dge_compact_paged(ctypes.byref(p), ctypes.byref(pg), 0x2000, ctypes.byref(t),
+                                 ctypes.byref(t), 0x3000, 0x4000, None, None) == code
+    assert lib.dge_compact_inplace_paged(ctypes.byref(p), ctypes.byref(pg), 0x2000,
+                                         ctypes.byref(t), ctypes.byref(t), None, None) == code
