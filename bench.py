@@ -50,6 +50,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--page-size", type=int, default=0,
+                    help="lay K and V out as a paged cache with pages of this many positions")
     ap.add_argument("--lse-supplied", action="store_true",
                     help="time the one-pass scoring with the row normalisers supplied "
                          "(dge_buffers.lse_in), computed once before the timed region")
@@ -94,6 +96,8 @@ def select_workload(args):
                       budgets=wl.budgets[:args.layers])
     if getattr(args, "lse_supplied", False):
         wl = wl.with_(name=f"{wl.name}+lse")
+    if getattr(args, "page_size", 0):
+        wl = wl.with_(name=f"{wl.name}+pages{args.page_size}")
     return wl
 
 
@@ -289,19 +293,28 @@ def run_ours(args):
     _build.build()
     wl = select_workload(args)
     tens = inputs.make_inputs(wl, device=device)
+    paging = None
+    if args.page_size:
+        # The same cache as page pools behind a block table (pages in a seeded random order).
+        K, bt = inputs.paged_layout(tens["K"], args.page_size, seed=1)
+        V, _ = inputs.paged_layout(tens["V"], args.page_size, seed=1)
+        tens = dict(tens, K=K, V=V, bt=bt)
+        paging = api.Paging(block_table=bt, page_size=args.page_size)
     p = api.problem_from_workload(wl)
     Q = tens["Q"] if wl.variant != inputs.STREAMING else None
     ws = api.workspace(p, device)
     if args.lse_supplied:
         # The row normalisers an attention pass over the observation rows would hand over;
         # here the library's own two-pass scoring computes them once, outside the timing.
-        tens = dict(tens, lse=api.evict(p, tens["K"], tens["V"], Q, ws=ws, want_lse=True)["lse"])
-    out = api.evict(p, tens["K"], tens["V"], Q, ws=ws, lse_in=tens.get("lse"))  # outputs once
+        tens = dict(tens, lse=api.evict(p, tens["K"], tens["V"], Q, ws=ws, want_lse=True,
+                                        paging=paging)["lse"])
+    out = api.evict(p, tens["K"], tens["V"], Q, ws=ws, lse_in=tens.get("lse"),
+                    paging=paging)  # outputs once
     stream = torch.cuda.current_stream(device)
 
     def step():
         api.evict(p, tens["K"], tens["V"], Q, ws=ws, out=out, stream=stream,
-                  lse_in=tens.get("lse"))
+                  lse_in=tens.get("lse"), paging=paging)
 
     for _ in range(args.warmup):
         step()
@@ -351,14 +364,14 @@ def run_ours(args):
             ach = flops / (per / 1e3) / 1e12
             roofline = {"bound": "tensor", "kernel": name, "achieved": round(ach, 1),
                         "peak": tflops, "unit": "TFLOP/s", "frac": round(ach / tflops, 4),
-                        "traffic": ncu_traffic(name, args.workload),
+                        "traffic": ncu_traffic(name, wl.name),
                         "alg_flops_per_launch": flops, "alg_bytes_per_launch": alg,
                         "peak_source": f"{peak_kind} bf16_tflops_sustained"}
         else:
             ach = alg / (per / 1e3) / 1e9
             roofline = {"bound": "hbm", "kernel": name, "achieved": round(ach, 1), "peak": hbm,
                         "unit": "GB/s", "frac": round(ach / hbm, 4),
-                        "traffic": ncu_traffic(name, args.workload),
+                        "traffic": ncu_traffic(name, wl.name),
                         "alg_bytes_per_launch": alg, "peak_source": f"{peak_kind} hbm_gbs"}
     step_gbs = step_bytes(wl) / (ms_step / 1e3) / 1e9
 
@@ -409,11 +422,15 @@ def run_e2e(args, wl, p, tens, out, ws, device, stream, world, api):
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
     d2h = sum(t.numel() * t.element_size() for t in host_out.values())
 
+    paging = None
+    if "bt" in dev_in:
+        paging = api.Paging(block_table=dev_in["bt"], page_size=dev_in["K"].shape[2])
+
     def step():
         for k in host_in:
             dev_in[k].copy_(host_in[k], non_blocking=True)
         api.evict(p, dev_in["K"], dev_in["V"], Q, ws=ws, out=out, stream=stream,
-                  lse_in=dev_in.get("lse"))
+                  lse_in=dev_in.get("lse"), paging=paging)
         for k in host_out:
             host_out[k].copy_(out[k], non_blocking=True)
 
@@ -439,8 +456,9 @@ def workload_text(wl):
     return (f"{wl.name}: L={wl.L} b={wl.b} Hq={wl.Hq} Hkv={wl.Hkv} d={wl.d} n={wl.n} "
             f"w={wl.w}+k={wl.k} {kind[wl.variant]}, {pool[wl.pool]}, {bud}, bf16 K/V/Q N(0,1), "
             f"sink x{wl.sink_scale:g}, {wl.n_spans} planted spans"
-            + (", row normalisers supplied (one pass over K)" if wl.name.endswith("+lse")
-               else ""))
+            + (", row normalisers supplied (one pass over K)" if "+lse" in wl.name else "")
+            + (f", paged cache ({wl.name.split('+pages')[1]}-position pages, block table)"
+               if "+pages" in wl.name else ""))
 
 
 # --- CPU oracle (baseline leg and reference arm) ----------------------------------------

@@ -106,7 +106,8 @@ __host__ __device__ inline size_t smem_bytes(int phase, int r_pad, int nslab)
            + (size_t)2 * nslab * stat_slab(phase, r_pad)        // stationary operand
            + (size_t)kStages * nslab * ring_slab(phase, r_pad)  // streamed operand
            + kCtrlBytes + (size_t)kLseSlots * kLseGroup * kLseBlock * 4
-           + (size_t)2 * kEpiWG * 4 * kMaxGroups * 16 * 4 + (size_t)kXchBufs * kEpiWG * kTile * 4;
+           + (size_t)2 * kEpiWG * 4 * kMaxGroups * 16 * 4 + (size_t)kXchBufs * kEpiWG * kTile * 4
+           + (size_t)tc::kPageWindow * 4;
 }
 
 struct Smem {
@@ -118,6 +119,7 @@ struct Smem {
     float *lse;        // [kLseSlots][kLseGroup][kLseBlock] -lse of streamed blocks (phase 2)
     float *red;        // [2][kEpiWG][4][kMaxGroups * 16] per-warp row sums (phase 1)
     float *xch;        // [kXchBufs][kEpiWG][128] per-warpgroup column sums (phase 2)
+    int *pages;        // [tc::kPageWindow] page ids of the producer's window (paged caches)
 };
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int phase, int r_pad, int nslab)
@@ -138,6 +140,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int phase, int r_pad, int ns
     s.red = reinterpret_cast<float *>(raw + off);
     off += 2 * kEpiWG * 4 * kMaxGroups * 16 * 4;
     s.xch = reinterpret_cast<float *>(raw + off);
+    off += kXchBufs * kEpiWG * kTile * 4;
+    s.pages = reinterpret_cast<int *>(raw + off);
     return s;
 }
 
@@ -348,14 +352,25 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                         ptx::tma_load_5d_hint(sdst + s * sslab, &tmQ, &sm.bar[kBarStatFull + sb],
                                               s * 64, T.blk * a.pb, h * g.G, bb, l, once_pol);
                     }
-                    if (a.phase == 2)
-                        tc::load_k_tile<kPaged>(sdst, sslab, a.nslab, &tmK, &sm.bar[kBarStatFull + sb],
-                                        T.blk * kTile, l, bb, h, a.kp, once_pol);
+                    if (a.phase == 2) {
+                        if constexpr (kPaged)
+                            tc::fetch_pages(sm.pages, a.kp, bb, T.blk * kTile, 1);
+                        tc::load_k_tile<kPaged>(sdst, sslab, a.nslab, &tmK,
+                                                &sm.bar[kBarStatFull + sb], T.blk * kTile, l, bb,
+                                                h, a.kp, sm.pages, T.blk * kTile, once_pol);
+                    }
                     if (++sb == 2) {
                         sb = 0;
                         sph ^= 1;
                     }
+                    int w0 = 0;   // first key of the page-id window (paged caches)
                     for (int i = 0; i < T.ntiles; ++i) {
+                        if constexpr (kPaged) {
+                            if (a.phase == 1 && i % tc::kPageWindowTiles == 0) {
+                                w0 = i * kTile;
+                                tc::fetch_pages(sm.pages, a.kp, bb, w0);
+                            }
+                        }
                         if (!wait(&sm.bar[kBarRingEmpty + rs], rph ^ 1)) {
                             ok = false;
                             break;
@@ -365,8 +380,9 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                                                    a.phase == 1 ? kbytes : qbytes);
                         flag[kFlagRingArm + rs] = (int)rph;
                         if (a.phase == 1)
-                            tc::load_k_tile<kPaged>(rdst, rslab, a.nslab, &tmK, &sm.bar[kBarRingFull + rs],
-                                            i * kTile, l, bb, h, a.kp, shared_pol);
+                            tc::load_k_tile<kPaged>(rdst, rslab, a.nslab, &tmK,
+                                                    &sm.bar[kBarRingFull + rs], i * kTile, l, bb,
+                                                    h, a.kp, sm.pages, w0, shared_pol);
                         else
                             for (int s = 0; s < a.nslab; ++s)
                                 ptx::tma_load_5d_hint(rdst + s * rslab, &tmQ,

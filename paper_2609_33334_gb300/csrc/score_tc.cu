@@ -181,6 +181,7 @@ struct Smem {
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
     float *xch;          // [kAccBufs][kEpiWG][128] phase-2 partial column sums
     int *xcnt;           // [kAccBufs][4] arrivals (row-block path: exactly one finaliser)
+    int *pages;          // [tc::kPageWindow] page ids of the producer's window (paged caches)
 };
 
 __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
@@ -191,7 +192,7 @@ __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
            + kStageBytes                          // lse merge staging
            + kCtrlBytes                           // barriers, tmem holder, flags
            + (2 * 256 + 2 * kEpiWG * 4 * kMaxGroups * 16) * 4 + 16
-           + kAccBufs * kEpiWG * kTile * 4 + kAccBufs * 4 * 4;
+           + kAccBufs * kEpiWG * kTile * 4 + kAccBufs * 4 * 4 + tc::kPageWindow * 4;
 }
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
@@ -221,6 +222,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int ks
     s.xch = reinterpret_cast<float *>(raw + off);
     off += kAccBufs * kEpiWG * kTile * 4;
     s.xcnt = reinterpret_cast<int *>(raw + off);
+    off += kAccBufs * 4 * 4;
+    s.pages = reinterpret_cast<int *>(raw + off);
     return s;
 }
 
@@ -427,7 +430,14 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     if (qb == 0)
                         qph ^= 1;
                     const uint64_t pol = T.phase == 2 ? drop : keep;
+                    int w0 = 0;   // first key of the page-id window (paged caches)
                     for (int tile = 0; tile < T.ntiles; ++tile) {
+                        if constexpr (kPaged) {
+                            if (tile % tc::kPageWindowTiles == 0) {
+                                w0 = T.k_lo + tile * kTile;
+                                tc::fetch_pages(sm.pages, a.kp, bb, w0);
+                            }
+                        }
                         c0 = tclock<kTr>();
                         if (!wait_bar(&sm.bar[kBarKEmpty + ks], kph ^ 1, flag, a)) {
                             ok = false;
@@ -438,9 +448,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         ptx::mbar_arrive_expect_tx(&sm.bar[kBarKFull + ks],
                                                    (uint32_t)a.nslab * kSlabBytes);
                         flag[kFlagKArm + ks] = (int)kph;
-                        tc::load_k_tile<kPaged>(sm.k + (size_t)ks * a.nslab * kSlabBytes, kSlabBytes,
-                                        a.nslab, &tmK, &sm.bar[kBarKFull + ks],
-                                        T.k_lo + tile * kTile, l, bb, h, a.kp, pol);
+                        tc::load_k_tile<kPaged>(sm.k + (size_t)ks * a.nslab * kSlabBytes,
+                                                kSlabBytes, a.nslab, &tmK, &sm.bar[kBarKFull + ks],
+                                                T.k_lo + tile * kTile, l, bb, h, a.kp, sm.pages,
+                                                w0, pol);
                         if (++ks == a.kstages) {
                             ks = 0;
                             kph ^= 1;

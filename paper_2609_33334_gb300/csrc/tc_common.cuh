@@ -97,44 +97,58 @@ struct KPaging {
 
 // Largest number of pages a 128-key tile spans (page sizes 16, 32, 64 or multiples of 128).
 constexpr int kMaxTilePages = 8;
+// Key tiles whose page ids are fetched together (kPageWindowTiles * kMaxTilePages ints of
+// shared memory).
+constexpr int kPageWindowTiles = 32;
+constexpr int kPageWindow = kPageWindowTiles * kMaxTilePages;
+
+// The page ids of positions [k0, min(k0 + tiles * 128, n)) of sequence bb (tiles <=
+// kPageWindowTiles) into shared memory with 4-byte asynchronous copies, waited for before
+// returning (one round trip a window); ids[i] belongs to page k0 / page_size + i.  Invalid
+// ids are clamped when read.
+__device__ __forceinline__ void fetch_pages(int *ids, const KPaging &pg, int bb, int k0,
+                                            int tiles = kPageWindowTiles)
+{
+    const int end = min(k0 + tiles * 128, pg.n);
+    const int p0 = k0 / pg.page_size, p1 = (end - 1) / pg.page_size;
+    const int32_t *src = pg.bt + (int64_t)bb * pg.pps;
+    for (int p = p0; p <= p1; ++p)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_addr(ids + (p - p0))),
+                     "l"(src + p)
+                     : "memory");
+    asm volatile("cp.async.wait_all;" ::: "memory");
+}
 
 // One 128-key tile of K (nslab slabs of 64 columns, slab_bytes apart) into shared memory with
 // TMA, completing on `bar`: one box per slab from a contiguous cache (map over
 // [L][b][Hkv][n][d]), or one box of min(page_size, 128) slots per page from a paged one (map
-// over [L][page][slot][Hkv][d]).  Page ids are all read before the first copy is issued (one
-// round trip a tile); positions past the cache read page 0, whose rows the callers mask.
+// over [L][page][slot][Hkv][d]; `ids` from fetch_pages for the window starting at `w0`).
+// Positions past the cache read page 0, whose rows the callers mask.
 template <bool kPaged>
 __device__ __forceinline__ void load_k_tile(uint8_t *dst, uint32_t slab_bytes, int nslab,
                                             const CUtensorMap *map, uint64_t *bar, int k0, int l,
-                                            int bb, int h, const KPaging &pg, uint64_t policy)
+                                            int bb, int h, const KPaging &pg, const int *ids,
+                                            int w0, uint64_t policy)
 {
     if constexpr (!kPaged) {
         for (int s = 0; s < nslab; ++s)
             ptx::tma_load_5d_hint(dst + s * slab_bytes, map, bar, s * 64, k0, h, bb, l, policy);
-        return;
-    }
-    else {
+    } else {
         const int rows = pg.page_size < 128 ? pg.page_size : 128;
         const int npg = 128 / rows;
-        int page[kMaxTilePages];
-#pragma unroll
-        for (int j = 0; j < kMaxTilePages; ++j) {
+        const int pbase = w0 / pg.page_size;
+        for (int j = 0; j < npg; ++j) {
             const int pos = k0 + j * rows;
-            page[j] = 0;
-            if (j < npg && pos < pg.n) {
-                const int pid = __ldg(pg.bt + (int64_t)bb * pg.pps + pos / pg.page_size);
-                page[j] = (pid >= 0 && pid < pg.num_pages) ? pid : 0;
+            int page = 0, slot = 0;
+            if (pos < pg.n) {
+                const int pid = ids[pos / pg.page_size - pbase];
+                page = (pid >= 0 && pid < pg.num_pages) ? pid : 0;
+                slot = pos % pg.page_size;
             }
+            for (int s = 0; s < nslab; ++s)
+                ptx::tma_load_5d_hint(dst + s * slab_bytes + j * rows * 128, map, bar, s * 64, h,
+                                      slot, page, l, policy);
         }
-#pragma unroll
-        for (int j = 0; j < kMaxTilePages; ++j)
-            if (j < npg) {
-                const int pos = k0 + j * rows;
-                const int slot = pos < pg.n ? pos % pg.page_size : 0;
-                for (int s = 0; s < nslab; ++s)
-                    ptx::tma_load_5d_hint(dst + s * slab_bytes + j * rows * 128, map, bar, s * 64,
-                                          h, slot, page[j], l, policy);
-            }
     }
 }
 
