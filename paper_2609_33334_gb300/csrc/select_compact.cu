@@ -79,18 +79,12 @@ __device__ __forceinline__ int64_t unit_row_base(const SelectParams &p, int64_t 
     return p.layers.row_base[l] + (int64_t)(bb * p.g.Hkv + h) * budget;
 }
 
-// Block-wide exclusive scan of one flag per thread (ballot + warp totals).
-// Returns this thread's exclusive prefix and writes the block total to *total.
-__device__ __forceinline__ int block_flag_scan(bool flag, int *warp_tot, int *total)
+// Exclusive scan of one int per warp (cnt[0..kSelWarps)) into base[], by warp 0.
+__device__ __forceinline__ void scan_warp_counts(const int *cnt, int *base)
 {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const unsigned bal = __ballot_sync(0xffffffffu, flag);
-    const int in_warp = __popc(bal & ((1u << lane) - 1u));
-    if (lane == 0)
-        warp_tot[warp] = __popc(bal);
-    __syncthreads();
-    if (warp == 0) {
-        const int v = lane < kSelWarps ? warp_tot[lane] : 0;
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        const int v = lane < kSelWarps ? cnt[lane] : 0;
         int incl = v;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
@@ -99,13 +93,163 @@ __device__ __forceinline__ int block_flag_scan(bool flag, int *warp_tot, int *to
                 incl += o;
         }
         if (lane < kSelWarps)
-            warp_tot[kSelWarps + lane] = incl - v;  // exclusive offset of warp `lane`
-        if (lane == 31)
-            *total = incl;
+            base[lane] = incl - v;
+    }
+}
+
+constexpr int kRadixBits = 11;
+constexpr int kRadixBins = 1 << kRadixBits;
+
+// Shared-memory scratch of the selection helpers.
+struct SelScratch {
+    uint32_t hist[kRadixBins];
+    int warp_a[kSelWarps], warp_b[kSelWarps], warp_c[kSelWarps];
+    uint32_t prefix;
+    int rank;
+};
+
+// T = the keep-th largest of the C keys key_at(0 .. C-1) (1 <= keep < C) and need_eq = how
+// many keys equal to T are kept (those at the lowest positions).  Radix select from the
+// highest bit in which the smallest and the largest key differ (the bits above are common to
+// every key), kRadixBits a pass: the scores of one unit share a few exponents, so histograms
+// of the top bits would put nearly every key in a handful of bins, whose shared-memory atomics
+// serialise.  Called by every thread of a block of kSelThreads.
+template <typename KeyAt>
+__device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, uint32_t &T,
+                                int &need_eq)
+{
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    uint32_t kmin = 0xffffffffu, kmax = 0u;
+    for (int j = tid; j < C; j += kSelThreads) {
+        const uint32_t k = key_at(j);
+        kmin = min(kmin, k);
+        kmax = max(kmax, k);
+    }
+    kmin = __reduce_min_sync(0xffffffffu, kmin);
+    kmax = __reduce_max_sync(0xffffffffu, kmax);
+    if (lane == 0) {
+        sc.warp_a[warp] = (int)kmin;
+        sc.warp_b[warp] = (int)kmax;
     }
     __syncthreads();
-    const int r = warp_tot[kSelWarps + warp] + in_warp;
-    return r;
+    if (warp == 0) {
+        const uint32_t a = __reduce_min_sync(0xffffffffu, (uint32_t)sc.warp_a[lane]);
+        const uint32_t b = __reduce_max_sync(0xffffffffu, (uint32_t)sc.warp_b[lane]);
+        if (lane == 0) {
+            sc.warp_c[0] = (int)a;
+            sc.warp_c[1] = (int)b;
+        }
+    }
+    __syncthreads();
+    kmin = (uint32_t)sc.warp_c[0];
+    kmax = (uint32_t)sc.warp_c[1];
+    const uint32_t diff = kmin ^ kmax;
+    const int top = diff ? 31 - __clz(diff) : -1;   // bits [0, top] vary
+    uint32_t mask = top >= 31 ? 0u : ~((2u << top) - 1u);
+    uint32_t prefix = kmax & mask;
+    int rank = keep;  // 1-based rank of T among the keys matching `prefix`, from the top
+    const int npass = (top + kRadixBits) / kRadixBits;
+#pragma unroll 1
+    for (int pass = 0; pass < npass; ++pass) {
+        const int hi = top - kRadixBits * pass;         // highest bit of this pass
+        const int shift = hi >= kRadixBits - 1 ? hi - (kRadixBits - 1) : 0;
+        const uint32_t bmask = (2u << (hi - shift)) - 1u;
+        for (int i = tid; i < kRadixBins; i += kSelThreads)
+            sc.hist[i] = 0;
+        __syncthreads();
+        for (int j = tid; j < C; j += kSelThreads) {
+            const uint32_t k = key_at(j);
+            if ((k & mask) == prefix)
+                atomicAdd(&sc.hist[(k >> shift) & bmask], 1u);
+        }
+        __syncthreads();
+        if (warp == 0) {
+            // Suffix counts over the bins, from the top: a lane sums kRadixBins / 32
+            // consecutive bins (bins above bmask are empty).
+            constexpr int per = kRadixBins / 32;
+            const int tb = kRadixBins - 1 - lane * per;   // this lane's bins: tb, tb-1, ...
+            uint32_t local = 0;
+            for (int q = 0; q < per; ++q)
+                local += sc.hist[tb - q];
+            uint32_t incl = local;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const uint32_t o = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off)
+                    incl += o;
+            }
+            uint32_t run = incl - local;
+            if (run < (uint32_t)rank && run + local >= (uint32_t)rank) {
+                for (int q = 0; q < per; ++q) {
+                    const uint32_t c = sc.hist[tb - q];
+                    if (run + c >= (uint32_t)rank) {
+                        sc.prefix = prefix | ((uint32_t)(tb - q) << shift);
+                        sc.rank = rank - (int)run;
+                        break;
+                    }
+                    run += c;
+                }
+            }
+        }
+        __syncthreads();
+        prefix = sc.prefix;
+        rank = sc.rank;
+        mask |= bmask << shift;
+        __syncthreads();
+    }
+    T = npass == 0 ? kmax : prefix;   // npass == 0: every key is equal
+    need_eq = rank;
+}
+
+// Writes the positions s0 + j of the kept keys -- every key above T and the first need_eq keys
+// equal to T -- in ascending order to out[0 .. keep).  Warp w walks a contiguous range of the
+// candidates twice: it counts its keys above and equal to T, then (after two scans over the
+// warps) writes its kept positions; the equal keys a warp keeps follow from the equal keys
+// before its range.  Called by every thread of a block of kSelThreads.
+template <typename KeyAt>
+__device__ void ordered_compaction(KeyAt key_at, int C, uint32_t T, int need_eq, int keep, int s0,
+                                   int32_t *out, SelScratch &sc)
+{
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint32_t lt_mask = (1u << lane) - 1u;
+    const int per_w = ((C + kSelWarps - 1) / kSelWarps + 31) & ~31;
+    const int w_lo = min(C, warp * per_w), w_hi = min(C, w_lo + per_w);
+    int eq_cnt = 0, gt_cnt = 0;
+    for (int c = w_lo; c < w_hi; c += 32) {
+        const int j = c + lane;
+        const uint32_t k = j < w_hi ? key_at(j) : 0u;
+        eq_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k == T));
+        gt_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k > T));
+    }
+    if (lane == 0) {
+        sc.warp_a[warp] = eq_cnt;
+        sc.warp_b[warp] = gt_cnt;
+    }
+    __syncthreads();
+    scan_warp_counts(sc.warp_a, sc.warp_c);
+    __syncthreads();
+    const int eq_base = sc.warp_c[warp];
+    const int eq_kept = min(eq_cnt, max(0, need_eq - eq_base));
+    __syncthreads();                      // every warp has read its equal-key offset
+    if (lane == 0)
+        sc.warp_a[warp] = sc.warp_b[warp] + eq_kept;
+    __syncthreads();
+    scan_warp_counts(sc.warp_a, sc.warp_c);
+    __syncthreads();
+    int sel_run = sc.warp_c[warp], eq_run = eq_base;
+    for (int c = w_lo; c < w_hi; c += 32) {
+        const int j = c + lane;
+        const uint32_t k = j < w_hi ? key_at(j) : 0u;
+        const bool eq = j < w_hi && k == T;
+        const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+        const bool sel = j < w_hi && (k > T || (eq && eq_run + __popc(eqb & lt_mask) < need_eq));
+        const uint32_t selb = __ballot_sync(0xffffffffu, sel);
+        const int pos = sel_run + __popc(selb & lt_mask);
+        if (sel && pos < keep)
+            out[pos] = s0 + j;
+        sel_run += __popc(selb);
+        eq_run += __popc(eqb);
+    }
 }
 
 template <bool SMEM>
@@ -113,11 +257,7 @@ __global__ void __launch_bounds__(kSelThreads)
 select_kernel(const float *__restrict__ scores, int32_t *__restrict__ idx, SelectParams p)
 {
     extern __shared__ __align__(16) uint32_t skeys[];
-    __shared__ uint32_t hist[256];
-    __shared__ int warp_tot[2 * kSelWarps];
-    __shared__ int s_total[2];
-    __shared__ uint32_t s_prefix;
-    __shared__ int s_rank;
+    __shared__ SelScratch scr;
 
     const int64_t u = blockIdx.x;
     const Geometry &g = p.g;
@@ -147,72 +287,10 @@ select_kernel(const float *__restrict__ scores, int32_t *__restrict__ idx, Selec
     }
     auto key_at = [&](int j) -> uint32_t { return SMEM ? skeys[j] : float_key(sc[j]); };
 
-    // Radix select, 8 bits per pass from the top: find T = the keep-th largest key.
-    uint32_t prefix = 0, mask = 0;
-    int rank = keep;  // 1-based rank of T among keys matching `prefix`, from the top
-    for (int shift = 24; shift >= 0; shift -= 8) {
-        if (threadIdx.x < 256)
-            hist[threadIdx.x] = 0;
-        __syncthreads();
-        for (int j = threadIdx.x; j < C; j += kSelThreads) {
-            const uint32_t k = key_at(j);
-            if ((k & mask) == prefix)
-                atomicAdd(&hist[(k >> shift) & 255u], 1u);
-        }
-        __syncthreads();
-        if (threadIdx.x < 32) {
-            // Suffix sums over bins 255..0 by one warp: lane handles 8 bins.
-            const int lane = threadIdx.x;
-            uint32_t c[8];
-            uint32_t local = 0;
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                c[q] = hist[255 - (lane * 8 + q)];
-                local += c[q];
-            }
-            uint32_t incl = local;
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const uint32_t o = __shfl_up_sync(0xffffffffu, incl, off);
-                if (lane >= off)
-                    incl += o;
-            }
-            uint32_t run = incl - local;  // keys in bins above this lane's first bin
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                if (run < (uint32_t)rank && run + c[q] >= (uint32_t)rank) {
-                    s_prefix = prefix | ((uint32_t)(255 - (lane * 8 + q)) << shift);
-                    s_rank = rank - (int)run;
-                }
-                run += c[q];
-            }
-        }
-        __syncthreads();
-        prefix = s_prefix;
-        rank = s_rank;
-        mask |= 255u << shift;
-        __syncthreads();
-    }
-    const uint32_t T = prefix;
-    const int need_eq = rank;  // keys equal to T to keep, lowest positions first
-
-    // Position-ordered compaction.
-    int sel_base = 0, eq_base = 0;
-    for (int base = 0; base < C; base += kSelThreads) {
-        const int j = base + threadIdx.x;
-        const uint32_t k = j < C ? key_at(j) : 0u;
-        const bool eq = j < C && k == T;
-        const int eq_rank = eq_base + block_flag_scan(eq, warp_tot, &s_total[0]);
-        const int eq_tot = s_total[0];
-        const bool sel = j < C && (k > T || (eq && eq_rank < need_eq));
-        const int pos = sel_base + block_flag_scan(sel, warp_tot, &s_total[1]);
-        const int sel_tot = s_total[1];
-        if (sel && pos < keep)
-            out[s0 + pos] = s0 + j;
-        eq_base += eq_tot;
-        sel_base += sel_tot;
-        __syncthreads();
-    }
+    uint32_t T;
+    int need_eq;
+    radix_threshold(key_at, C, keep, scr, T, need_eq);
+    ordered_compaction(key_at, C, T, need_eq, keep, s0, out + s0, scr);
 }
 
 cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const float *scores,
@@ -249,25 +327,7 @@ cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const flo
 constexpr int kPsThreads = 1024;
 constexpr int kPsPer = 32;                       // positions pooled per thread (registers)
 constexpr int kPsMaxP = kPsThreads * kPsPer;     // 32768
-constexpr int kPsBins = 2048;                    // radix bins (11 bits)
 
-// Exclusive scan of one int per warp (cnt[0..kSelWarps)) into base[], by warp 0.
-__device__ __forceinline__ void scan_warp_counts(const int *cnt, int *base)
-{
-    if (threadIdx.x < 32) {
-        const int lane = threadIdx.x;
-        const int v = lane < kSelWarps ? cnt[lane] : 0;
-        int incl = v;
-#pragma unroll
-        for (int off = 1; off < 32; off <<= 1) {
-            const int o = __shfl_up_sync(0xffffffffu, incl, off);
-            if (lane >= off)
-                incl += o;
-        }
-        if (lane < kSelWarps)
-            base[lane] = incl - v;
-    }
-}
 
 // Pooled value at position j of a row of P raw scores in shared memory.  R > 0: the pool
 // radius known at compile time (interior positions unrolled); R < 0: radius r at run time.
@@ -296,13 +356,9 @@ pool_select_kernel(const float *__restrict__ raw, float *__restrict__ pooled_out
                    int32_t *__restrict__ idx, SelectParams p, int kernel)
 {
     extern __shared__ __align__(16) uint32_t sbuf[];  // [P]: raw scores, then pooled keys
-    __shared__ uint32_t hist[kPsBins];
-    __shared__ int warp_cnt[kSelWarps], warp_base[kSelWarps], warp_gt[kSelWarps];
-    __shared__ uint32_t s_prefix;
-    __shared__ int s_rank;
+    __shared__ SelScratch sc;
 
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const uint32_t lt_mask = (1u << lane) - 1u;
+    const int tid = threadIdx.x;
     const int64_t u = blockIdx.x;
     const Geometry &g = p.g;
     int budget;
@@ -348,100 +404,11 @@ pool_select_kernel(const float *__restrict__ raw, float *__restrict__ pooled_out
         return;
     }
     const uint32_t *keys = sbuf + s0;
-
-    // Radix select from the top, 11 + 11 + 10 bits: T = the keep-th largest key.
-    uint32_t prefix = 0, mask = 0;
-    int rank = keep;
-#pragma unroll 1
-    for (int pass = 0; pass < 3; ++pass) {
-        const int shift = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
-        const uint32_t bmask = pass == 2 ? 1023u : 2047u;
-        for (int i = tid; i < kPsBins; i += kPsThreads)
-            hist[i] = 0;
-        __syncthreads();
-        for (int j = tid; j < C; j += kPsThreads) {
-            const uint32_t k = keys[j];
-            if ((k & mask) == prefix)
-                atomicAdd(&hist[(k >> shift) & bmask], 1u);
-        }
-        __syncthreads();
-        if (tid < 32) {
-            // Suffix counts over the bins, from the top: lane handles 64 consecutive bins.
-            const int nb = (int)bmask + 1, per = nb / 32;
-            const int top = nb - 1 - lane * per;   // this lane's bins: top, top-1, ...
-            uint32_t local = 0;
-            for (int q = 0; q < per; ++q)
-                local += hist[top - q];
-            uint32_t incl = local;
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const uint32_t o = __shfl_up_sync(0xffffffffu, incl, off);
-                if (lane >= off)
-                    incl += o;
-            }
-            uint32_t run = incl - local;
-            if (run < (uint32_t)rank && run + local >= (uint32_t)rank) {
-                for (int q = 0; q < per; ++q) {
-                    const uint32_t c = hist[top - q];
-                    if (run + c >= (uint32_t)rank) {
-                        s_prefix = prefix | ((uint32_t)(top - q) << shift);
-                        s_rank = rank - (int)run;
-                        break;
-                    }
-                    run += c;
-                }
-            }
-        }
-        __syncthreads();
-        prefix = s_prefix;
-        rank = s_rank;
-        mask |= bmask << shift;
-        __syncthreads();
-    }
-    const uint32_t T = prefix;
-    const int need_eq = rank;  // keys equal to T to keep, lowest positions first
-
-    // Position-ordered compaction: warp w owns candidates [w_lo, w_hi).  Pass 1 counts the
-    // keys above and equal to T; the warp keeps its keys above T and the equal keys whose
-    // rank among all equal keys is below need_eq.
-    const int per_w = ((C + kSelWarps - 1) / kSelWarps + 31) & ~31;
-    const int w_lo = min(C, warp * per_w), w_hi = min(C, w_lo + per_w);
-    int eq_cnt = 0, gt_cnt = 0;
-    for (int c = w_lo; c < w_hi; c += 32) {
-        const int j = c + lane;
-        const uint32_t k = j < w_hi ? keys[j] : 0u;
-        eq_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k == T));
-        gt_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k > T));
-    }
-    if (lane == 0) {
-        warp_cnt[warp] = eq_cnt;
-        warp_gt[warp] = gt_cnt;
-    }
-    __syncthreads();
-    scan_warp_counts(warp_cnt, warp_base);
-    __syncthreads();
-    const int eq_base = warp_base[warp];
-    const int eq_kept = min(eq_cnt, max(0, need_eq - eq_base));
-    __syncthreads();                      // every warp has read its equal-key offset
-    if (lane == 0)
-        warp_cnt[warp] = warp_gt[warp] + eq_kept;
-    __syncthreads();
-    scan_warp_counts(warp_cnt, warp_base);
-    __syncthreads();
-    int sel_run = warp_base[warp], eq_run = eq_base;
-    for (int c = w_lo; c < w_hi; c += 32) {
-        const int j = c + lane;
-        const uint32_t k = j < w_hi ? keys[j] : 0u;
-        const bool eq = j < w_hi && k == T;
-        const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
-        const bool sel = j < w_hi && (k > T || (eq && eq_run + __popc(eqb & lt_mask) < need_eq));
-        const uint32_t selb = __ballot_sync(0xffffffffu, sel);
-        const int pos = sel_run + __popc(selb & lt_mask);
-        if (sel && pos < keep)
-            out[s0 + pos] = s0 + j;
-        sel_run += __popc(selb);
-        eq_run += __popc(eqb);
-    }
+    auto key_at = [&](int j) -> uint32_t { return keys[j]; };
+    uint32_t T;
+    int need_eq;
+    radix_threshold(key_at, C, keep, sc, T, need_eq);
+    ordered_compaction(key_at, C, T, need_eq, keep, s0, out + s0, sc);
 }
 
 bool pool_select_supported(const Geometry &g) { return g.P <= kPsMaxP; }
