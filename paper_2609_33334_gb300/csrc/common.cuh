@@ -151,10 +151,11 @@ __device__ __forceinline__ void set_status(uint32_t *status, uint32_t code)
         atomicCAS(status, 0u, code);
 }
 
-// Order-preserving map of a float to uint32 (larger float -> larger key).
+// Order-preserving map of a float to uint32 (larger float -> larger key); -0.0 maps to the
+// key of +0.0, since the two compare equal (a tie broken by position, like any other).
 __device__ __forceinline__ uint32_t float_key(float f)
 {
-    const uint32_t u = __float_as_uint(f);
+    const uint32_t u = __float_as_uint(f == 0.f ? 0.f : f);
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
