@@ -52,6 +52,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--page-size", type=int, default=0,
                     help="lay K and V out as a paged cache with pages of this many positions")
+    ap.add_argument("--page-head-major", action="store_true",
+                    help="paged pools as [page][head][slot][d] instead of [page][slot][head][d]")
     ap.add_argument("--lse-supplied", action="store_true",
                     help="time the one-pass scoring with the row normalisers supplied "
                          "(dge_buffers.lse_in), computed once before the timed region")
@@ -97,7 +99,8 @@ def select_workload(args):
     if getattr(args, "lse_supplied", False):
         wl = wl.with_(name=f"{wl.name}+lse")
     if getattr(args, "page_size", 0):
-        wl = wl.with_(name=f"{wl.name}+pages{args.page_size}")
+        hm = "h" if getattr(args, "page_head_major", False) else ""
+        wl = wl.with_(name=f"{wl.name}+pages{args.page_size}{hm}")
     return wl
 
 
@@ -296,10 +299,11 @@ def run_ours(args):
     paging = None
     if args.page_size:
         # The same cache as page pools behind a block table (pages in a seeded random order).
-        K, bt = inputs.paged_layout(tens["K"], args.page_size, seed=1)
-        V, _ = inputs.paged_layout(tens["V"], args.page_size, seed=1)
+        hm = args.page_head_major
+        K, bt = inputs.paged_layout(tens["K"], args.page_size, seed=1, head_major=hm)
+        V, _ = inputs.paged_layout(tens["V"], args.page_size, seed=1, head_major=hm)
         tens = dict(tens, K=K, V=V, bt=bt)
-        paging = api.Paging(block_table=bt, page_size=args.page_size)
+        paging = api.Paging(block_table=bt, page_size=args.page_size, head_major=hm)
     p = api.problem_from_workload(wl)
     Q = tens["Q"] if wl.variant != inputs.STREAMING else None
     ws = api.workspace(p, device)
@@ -424,7 +428,9 @@ def run_e2e(args, wl, p, tens, out, ws, device, stream, world, api):
 
     paging = None
     if "bt" in dev_in:
-        paging = api.Paging(block_table=dev_in["bt"], page_size=dev_in["K"].shape[2])
+        hm = args.page_head_major
+        paging = api.Paging(block_table=dev_in["bt"],
+                            page_size=dev_in["K"].shape[3 if hm else 2], head_major=hm)
 
     def step():
         for k in host_in:
@@ -457,7 +463,8 @@ def workload_text(wl):
             f"w={wl.w}+k={wl.k} {kind[wl.variant]}, {pool[wl.pool]}, {bud}, bf16 K/V/Q N(0,1), "
             f"sink x{wl.sink_scale:g}, {wl.n_spans} planted spans"
             + (", row normalisers supplied (one pass over K)" if "+lse" in wl.name else "")
-            + (f", paged cache ({wl.name.split('+pages')[1]}-position pages, block table)"
+            + (f", paged cache ({wl.name.split('+pages')[1].rstrip('h')}-position pages"
+               + (", head-major" if wl.name.endswith("h") else "") + ", block table)"
                if "+pages" in wl.name else ""))
 
 

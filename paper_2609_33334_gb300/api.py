@@ -73,18 +73,21 @@ class Problem:
 @dataclasses.dataclass
 class Paging:
     """A paged cache (dge_paging): K and V are then pools [L][num_pages][page_size][Hkv][d]
-    and position p of sequence b lives in slot p % page_size of page
-    block_table[b, p // page_size] (int32 [b][pages_per_seq] on the device)."""
+    (``head_major``: [L][num_pages][Hkv][page_size][d]) and position p of sequence b lives in
+    slot p % page_size of page block_table[b, p // page_size] (int32 [b][pages_per_seq] on the
+    device)."""
 
     block_table: torch.Tensor
     page_size: int
+    head_major: bool = False
 
     def c(self, pool: torch.Tensor) -> B.dge_paging:
         bt = self.block_table
         if bt.dtype != torch.int32 or not bt.is_contiguous() or bt.dim() != 2:
             raise ValueError("block_table must be a contiguous int32 [b][pages_per_seq] tensor")
-        if pool.dim() != 5 or pool.shape[2] != self.page_size:
-            raise ValueError("paged K / V must be [L][num_pages][page_size][Hkv][d]")
+        if pool.dim() != 5 or pool.shape[3 if self.head_major else 2] != self.page_size:
+            raise ValueError("paged K / V must be [L][num_pages][page_size][Hkv][d] "
+                             "([L][num_pages][Hkv][page_size][d] when head_major)")
         return B.dge_paging(block_table=bt.data_ptr(), page_size=self.page_size,
                             pages_per_seq=bt.shape[1], num_pages=pool.shape[1],
                             stride_page=pool.stride(1))
@@ -95,9 +98,10 @@ def _kv_desc(t: torch.Tensor, paging: Optional[Paging]) -> B.dge_tensor:
         return B.tensor_desc(t)
     if t.dim() != 5 or t.stride(-1) != 1:
         raise ValueError("expected a 5-D pool with a contiguous last dim")
-    s = t.stride()   # [L][page][slot][head][d]
+    s = t.stride()   # [L][page][slot][head][d], or [L][page][head][slot][d] when head-major
+    head, slot = (s[2], s[3]) if paging.head_major else (s[3], s[2])
     return B.dge_tensor(data=t.data_ptr(), stride_layer=s[0], stride_batch=0,
-                        stride_head=s[3], stride_pos=s[2])
+                        stride_head=head, stride_pos=slot)
 
 
 def _paging_ptr(paging: Optional[Paging], pool: torch.Tensor):

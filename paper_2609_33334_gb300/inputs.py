@@ -210,10 +210,10 @@ def bf16_bits(t: torch.Tensor) -> np.ndarray:
 
 
 def paged_layout(cache: torch.Tensor, page_size: int, seed: int = 0, spare_pages: int = 3,
-                 extra_table_pages: int = 1) -> tuple:
+                 extra_table_pages: int = 1, head_major: bool = False) -> tuple:
     """Lay a contiguous cache [L][b][Hkv][n][d] out as a paged one, the way a paged-attention
-    server keeps it: returns (pool [L][num_pages][page_size][Hkv][d], block_table int32
-    [b][pages_per_seq]).  Sequences get pages in a seeded random order (shared by all
+    server keeps it: returns (pool [L][num_pages][page_size][Hkv][d], or with ``head_major``
+    [L][num_pages][Hkv][page_size][d], and block_table int32 [b][pages_per_seq]).  Sequences get pages in a seeded random order (shared by all
     layers), the pool has ``spare_pages`` pages no sequence uses, and the table has
     ``extra_table_pages`` entries per sequence past the cache (set to -1).  Every slot that
     holds no cache position is NaN, so a read of one shows in the results.  Pure layout: no
@@ -226,25 +226,34 @@ def paged_layout(cache: torch.Tensor, page_size: int, seed: int = 0, spare_pages
     perm = rng.permutation(num_pages)[:b * used].reshape(b, used)
     table = np.full((b, pps), -1, dtype=np.int32)
     table[:, :used] = perm
-    pool = torch.full((L, num_pages, page_size, Hkv, d), float("nan"), dtype=cache.dtype,
-                      device=cache.device)
+    shape = (L, num_pages, Hkv, page_size, d) if head_major else (L, num_pages, page_size, Hkv, d)
+    pool = torch.full(shape, float("nan"), dtype=cache.dtype, device=cache.device)
     for s in range(b):
         for j in range(used):
             lo, hi = j * page_size, min((j + 1) * page_size, n)
-            # [L][Hkv][rows][d] -> [L][rows][Hkv][d]
-            pool[:, int(perm[s, j]), :hi - lo] = cache[:, s, :, lo:hi].permute(0, 2, 1, 3)
+            if head_major:
+                pool[:, int(perm[s, j]), :, :hi - lo] = cache[:, s, :, lo:hi]
+            else:
+                # [L][Hkv][rows][d] -> [L][rows][Hkv][d]
+                pool[:, int(perm[s, j]), :hi - lo] = cache[:, s, :, lo:hi].permute(0, 2, 1, 3)
     return pool, torch.from_numpy(table).to(cache.device)
 
 
-def unpaged(pool: torch.Tensor, block_table: torch.Tensor, n: int) -> torch.Tensor:
+def unpaged(pool: torch.Tensor, block_table: torch.Tensor, n: int,
+            head_major: bool = False) -> torch.Tensor:
     """The contiguous cache [L][b][Hkv][n][d] that a paged one holds (inverse of paged_layout
     on positions [0, n))."""
-    L, _, page_size, Hkv, d = pool.shape
+    if head_major:
+        L, _, Hkv, page_size, d = pool.shape
+    else:
+        L, _, page_size, Hkv, d = pool.shape
     b = block_table.shape[0]
     out = torch.empty((L, b, Hkv, n, d), dtype=pool.dtype, device=pool.device)
     table = block_table.cpu().numpy()
     for s in range(b):
         for j in range((n + page_size - 1) // page_size):
             lo, hi = j * page_size, min((j + 1) * page_size, n)
-            out[:, s, :, lo:hi] = pool[:, int(table[s, j]), :hi - lo].permute(0, 2, 1, 3)
+            page = pool[:, int(table[s, j])]
+            out[:, s, :, lo:hi] = page[:, :, :hi - lo] if head_major else \
+                page[:, :hi - lo].permute(0, 2, 1, 3)
     return out

@@ -33,11 +33,11 @@ def built():
     _build.build()
 
 
-def _paged(tens, page_size, seed=0):
-    K, bt = inputs.paged_layout(tens["K"], page_size, seed=seed)
-    V, bt2 = inputs.paged_layout(tens["V"], page_size, seed=seed)
+def _paged(tens, page_size, seed=0, head_major=False):
+    K, bt = inputs.paged_layout(tens["K"], page_size, seed=seed, head_major=head_major)
+    V, bt2 = inputs.paged_layout(tens["V"], page_size, seed=seed, head_major=head_major)
     assert torch.equal(bt, bt2)
-    return K, V, api.Paging(block_table=bt, page_size=page_size)
+    return K, V, api.Paging(block_table=bt, page_size=page_size, head_major=head_major)
 
 
 def _q(wl, tens):
@@ -156,3 +156,31 @@ def test_paged_diagnostics_heldout():
     torch.cuda.synchronize()
     for k in a:
         assert torch.equal(a[k], b[k]), k
+
+
+@pytest.mark.parametrize("page_size", [16, 128])
+@pytest.mark.parametrize("name", ["c2_small", "c4_small", "slm_small"])
+def test_head_major_pages(name, page_size):
+    """Pools laid out [page][head][slot][d] (each head's page contiguous) through the same
+    strides: identical outputs, and the in-place gather writes the right slots."""
+    wl = CASES[name]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    want = wl.variant != inputs.STREAMING
+    ref = api.evict(p, tens["K"], tens["V"], _q(wl, tens), want_scores=want)
+    K, V, pg = _paged(tens, page_size, seed=3, head_major=True)
+    got = api.evict(p, K, V, _q(wl, tens), want_scores=want, paging=pg)
+    torch.cuda.synchronize()
+    for k in ("idx", "Kc", "Vc") + (("scores",) if want else ()):
+        assert torch.equal(got[k], ref[k]), k
+    api.evict_inplace(p, K, V, _q(wl, tens), paging=pg)
+    torch.cuda.synchronize()
+    Kn = inputs.unpaged(K, pg.block_table, wl.n, head_major=True)
+    offs = p.unit_row_offsets()
+    u = 0
+    for l in range(wl.L):
+        B = wl.budgets[l]
+        for b in range(wl.b):
+            for h in range(wl.Hkv):
+                assert torch.equal(Kn[l, b, h, :B], ref["Kc"][offs[u]:offs[u] + B])
+                u += 1
