@@ -54,6 +54,8 @@ def parse_args():
                     help="lay K and V out as a paged cache with pages of this many positions")
     ap.add_argument("--page-head-major", action="store_true",
                     help="paged pools as [page][head][slot][d] instead of [page][slot][head][d]")
+    ap.add_argument("--page-order", default="random", choices=["random", "sequential", "runs"],
+                    help="order in which sequences get their pages")
     ap.add_argument("--lse-supplied", action="store_true",
                     help="time the one-pass scoring with the row normalisers supplied "
                          "(dge_buffers.lse_in), computed once before the timed region")
@@ -100,7 +102,9 @@ def select_workload(args):
         wl = wl.with_(name=f"{wl.name}+lse")
     if getattr(args, "page_size", 0):
         hm = "h" if getattr(args, "page_head_major", False) else ""
-        wl = wl.with_(name=f"{wl.name}+pages{args.page_size}{hm}")
+        order = getattr(args, "page_order", "random")
+        wl = wl.with_(name=f"{wl.name}+pages{args.page_size}{hm}"
+                           + ("" if order == "random" else f"-{order}"))
     return wl
 
 
@@ -300,8 +304,10 @@ def run_ours(args):
     if args.page_size:
         # The same cache as page pools behind a block table (pages in a seeded random order).
         hm = args.page_head_major
-        K, bt = inputs.paged_layout(tens["K"], args.page_size, seed=1, head_major=hm)
-        V, _ = inputs.paged_layout(tens["V"], args.page_size, seed=1, head_major=hm)
+        K, bt = inputs.paged_layout(tens["K"], args.page_size, seed=1, head_major=hm,
+                                    order=args.page_order)
+        V, _ = inputs.paged_layout(tens["V"], args.page_size, seed=1, head_major=hm,
+                                   order=args.page_order)
         tens = dict(tens, K=K, V=V, bt=bt)
         paging = api.Paging(block_table=bt, page_size=args.page_size, head_major=hm)
     p = api.problem_from_workload(wl)
@@ -463,9 +469,14 @@ def workload_text(wl):
             f"w={wl.w}+k={wl.k} {kind[wl.variant]}, {pool[wl.pool]}, {bud}, bf16 K/V/Q N(0,1), "
             f"sink x{wl.sink_scale:g}, {wl.n_spans} planted spans"
             + (", row normalisers supplied (one pass over K)" if "+lse" in wl.name else "")
-            + (f", paged cache ({wl.name.split('+pages')[1].rstrip('h')}-position pages"
-               + (", head-major" if wl.name.endswith("h") else "") + ", block table)"
-               if "+pages" in wl.name else ""))
+            + (paged_text(wl.name.split("+pages")[1]) if "+pages" in wl.name else ""))
+
+
+def paged_text(tag):
+    size, _, order = tag.partition("-")
+    head = size.endswith("h")
+    return (f", paged cache ({size.rstrip('h')}-position pages" + (", head-major" if head else "")
+            + f", {order or 'random'} page order, block table)")
 
 
 # --- CPU oracle (baseline leg and reference arm) ----------------------------------------

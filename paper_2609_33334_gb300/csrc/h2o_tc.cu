@@ -25,6 +25,7 @@
 // DGE_ERR_DEVICE_TIMEOUT, stops issuing work, drains its own copies and MMAs and frees TMEM.
 #include <cuda.h>
 #include <math.h>
+#include <string.h>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -107,7 +108,7 @@ __host__ __device__ inline size_t smem_bytes(int phase, int r_pad, int nslab)
            + (size_t)kStages * nslab * ring_slab(phase, r_pad)  // streamed operand
            + kCtrlBytes + (size_t)kLseSlots * kLseGroup * kLseBlock * 4
            + (size_t)2 * kEpiWG * 4 * kMaxGroups * 16 * 4 + (size_t)kXchBufs * kEpiWG * kTile * 4
-           + (size_t)tc::kPageWindow * 4;
+           + (size_t)(tc::kPageWindow + 4) * 4;
 }
 
 struct Smem {
@@ -250,7 +251,7 @@ __device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
 template <bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
 h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
-              const H2oArgs a)
+              const __grid_constant__ CUtensorMap tmKm, const H2oArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     const Smem sm = carve(smem_raw, a.phase, a.r_pad, a.nslab);
@@ -353,22 +354,25 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                                               s * 64, T.blk * a.pb, h * g.G, bb, l, once_pol);
                     }
                     if (a.phase == 2) {
+                        const int *ids = sm.pages;
                         if constexpr (kPaged)
-                            tc::fetch_pages(sm.pages, a.kp, bb, T.blk * kTile, 1);
-                        tc::load_k_tile<kPaged>(sdst, sslab, a.nslab, &tmK,
+                            ids = tc::fetch_pages(sm.pages, a.kp, bb, T.blk * kTile, 1);
+                        tc::load_k_tile<kPaged>(sdst, sslab, a.nslab, &tmK, &tmKm,
                                                 &sm.bar[kBarStatFull + sb], T.blk * kTile, l, bb,
-                                                h, a.kp, sm.pages, T.blk * kTile, once_pol);
+                                                h, a.kp, ids, T.blk * kTile, once_pol);
                     }
                     if (++sb == 2) {
                         sb = 0;
                         sph ^= 1;
                     }
-                    int w0 = 0;   // first key of the page-id window (paged caches)
+                    int w0 = 0;               // first key of the page-id window (paged caches)
+                    const int *ids = sm.pages;
                     for (int i = 0; i < T.ntiles; ++i) {
                         if constexpr (kPaged) {
                             if (a.phase == 1 && i % tc::kPageWindowTiles == 0) {
                                 w0 = i * kTile;
-                                tc::fetch_pages(sm.pages, a.kp, bb, w0);
+                                ids = tc::fetch_pages(sm.pages, a.kp, bb, w0,
+                                                      min(T.ntiles - i, tc::kPageWindowTiles));
                             }
                         }
                         if (!wait(&sm.bar[kBarRingEmpty + rs], rph ^ 1)) {
@@ -380,9 +384,9 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                                                    a.phase == 1 ? kbytes : qbytes);
                         flag[kFlagRingArm + rs] = (int)rph;
                         if (a.phase == 1)
-                            tc::load_k_tile<kPaged>(rdst, rslab, a.nslab, &tmK,
+                            tc::load_k_tile<kPaged>(rdst, rslab, a.nslab, &tmK, &tmKm,
                                                     &sm.bar[kBarRingFull + rs], i * kTile, l, bb,
-                                                    h, a.kp, sm.pages, w0, shared_pol);
+                                                    h, a.kp, ids, w0, shared_pol);
                         else
                             for (int s = 0; s < a.nslab; ++s)
                                 ptx::tma_load_5d_hint(rdst + s * rslab, &tmQ,
@@ -806,7 +810,9 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
                           const H2oPlan &plan, float *lse2, float *raw, uint32_t *ready,
                           uint32_t *status, cudaStream_t stream, bool *encoded)
 {
-    CUtensorMap tmK, tmQ;
+    CUtensorMap tmK, tmQ, tmKm;
+    memset(&tmKm, 0, sizeof tmKm);
+    const bool merged = K.bt && tc::encode_k_merged_map(&tmKm, K, g.L, g.Hkv, g.d);
     *encoded = tc::encode_k_map(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d) &&
                tc::encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.n, g.d, plan.pb, g.G);
     if (!*encoded)
@@ -821,6 +827,7 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
     H2oArgs a;
     a.g = g;
     a.kp = tc::k_paging(K, g.n);
+    a.kp.merged = merged ? 1 : 0;
     a.phase = phase;
     a.pb = plan.pb;
     a.rows = plan.rows;
@@ -849,7 +856,7 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
     if (err != cudaSuccess)
         return err;
     const int64_t grid = a.items < sms ? a.items : sms;
-    kernel<<<(unsigned)grid, kThreads, smem, stream>>>(tmK, tmQ, a);
+    kernel<<<(unsigned)grid, kThreads, smem, stream>>>(tmK, tmQ, tmKm, a);
     return cudaGetLastError();
 }
 

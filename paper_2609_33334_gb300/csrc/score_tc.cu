@@ -29,6 +29,7 @@
 // frees TMEM and returns.
 #include <cuda.h>
 #include <math.h>
+#include <string.h>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -181,7 +182,7 @@ struct Smem {
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
     float *xch;          // [kAccBufs][kEpiWG][128] phase-2 partial column sums
     int *xcnt;           // [kAccBufs][4] arrivals (row-block path: exactly one finaliser)
-    int *pages;          // [tc::kPageWindow] page ids of the producer's window (paged caches)
+    int *pages;          // [tc::kPageWindow + 4] page ids of the producer's window (paged caches)
 };
 
 __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
@@ -192,7 +193,7 @@ __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
            + kStageBytes                          // lse merge staging
            + kCtrlBytes                           // barriers, tmem holder, flags
            + (2 * 256 + 2 * kEpiWG * 4 * kMaxGroups * 16) * 4 + 16
-           + kAccBufs * kEpiWG * kTile * 4 + kAccBufs * 4 * 4 + tc::kPageWindow * 4;
+           + kAccBufs * kEpiWG * kTile * 4 + kAccBufs * 4 * 4 + (tc::kPageWindow + 4) * 4;
 }
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
@@ -322,7 +323,7 @@ __device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
 template <bool kTr, bool kFx, bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
 score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
-                const TcArgs a)
+                const __grid_constant__ CUtensorMap tmKm, const TcArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     const Smem sm = carve(smem_raw, a.r_pad, a.nslab, a.kstages);
@@ -412,6 +413,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         continue;
                     int l, bb, h;
                     unit_coords(g, kFx ? T.u / a.nrb : T.u, l, bb, h);
+
                     const int qhead = h * g.G + (kFx ? (int)(T.u % a.nrb) * a.gsub : 0);
                     long long c0 = tclock<kTr>();
                     if (!wait_bar(&sm.bar[kBarQEmpty + qb], qph ^ 1, flag, a)) {
@@ -430,12 +432,14 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     if (qb == 0)
                         qph ^= 1;
                     const uint64_t pol = T.phase == 2 ? drop : keep;
-                    int w0 = 0;   // first key of the page-id window (paged caches)
+                    int w0 = 0;               // first key of the page-id window (paged caches)
+                    const int *ids = sm.pages;
                     for (int tile = 0; tile < T.ntiles; ++tile) {
                         if constexpr (kPaged) {
                             if (tile % tc::kPageWindowTiles == 0) {
                                 w0 = T.k_lo + tile * kTile;
-                                tc::fetch_pages(sm.pages, a.kp, bb, w0);
+                                ids = tc::fetch_pages(sm.pages, a.kp, bb, w0,
+                                                      min(T.ntiles - tile, tc::kPageWindowTiles));
                             }
                         }
                         c0 = tclock<kTr>();
@@ -449,8 +453,9 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                                                    (uint32_t)a.nslab * kSlabBytes);
                         flag[kFlagKArm + ks] = (int)kph;
                         tc::load_k_tile<kPaged>(sm.k + (size_t)ks * a.nslab * kSlabBytes,
-                                                kSlabBytes, a.nslab, &tmK, &sm.bar[kBarKFull + ks],
-                                                T.k_lo + tile * kTile, l, bb, h, a.kp, sm.pages,
+                                                kSlabBytes, a.nslab, &tmK, &tmKm,
+                                                &sm.bar[kBarKFull + ks],
+                                                T.k_lo + tile * kTile, l, bb, h, a.kp, ids,
                                                 w0, pol);
                         if (++ks == a.kstages) {
                             ks = 0;
@@ -1058,6 +1063,33 @@ bool encode_k_map(CUtensorMap *map, const TensorDesc &t, int L, int b, int Hkv, 
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Slots of consecutive pages adjacent in memory: page stride = page_size * slot stride.
+static bool slots_run_on(const TensorDesc &t)
+{
+    return t.bt && t.s_page == (int64_t)t.page_size * t.s_pos;
+}
+
+bool encode_k_merged_map(CUtensorMap *map, const TensorDesc &t, int L, int Hkv, int d)
+{
+    Encode fn = encode_fn_impl();
+    if (!fn || !slots_run_on(t))
+        return false;
+    // [L][slot over all pages][head][d], plus a unit outer dimension.
+    const int64_t slots = (int64_t)t.num_pages * t.page_size;
+    const int64_t s_layer = t.s_layer != 0 ? t.s_layer : t.s_page * t.num_pages;
+    const cuuint64_t dims[5] = {(cuuint64_t)d, (cuuint64_t)Hkv, (cuuint64_t)slots, (cuuint64_t)L, 1};
+    const cuuint64_t strides[4] = {(cuuint64_t)t.s_head * 2, (cuuint64_t)t.s_pos * 2,
+                                   (cuuint64_t)s_layer * 2, (cuuint64_t)s_layer * L * 2};
+    const cuuint32_t box[5] = {64, 1, 128, 1, 1};
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    for (int i = 0; i < 4; ++i)
+        if (strides[i] == 0 || strides[i] % 16 != 0)
+            return false;
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<__nv_bfloat16 *>(t.data), dims,
+              strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 KPaging k_paging(const TensorDesc &t, int n)
 {
     KPaging p;
@@ -1066,6 +1098,10 @@ KPaging k_paging(const TensorDesc &t, int n)
     p.pps = t.pps;
     p.num_pages = t.num_pages;
     p.n = n;
+    p.merged = 0;
+    p.ps_shift = 0;
+    while (p.ps_shift < 30 && (1 << p.ps_shift) < t.page_size)
+        ++p.ps_shift;
     return p;
 }
 
@@ -1146,7 +1182,9 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
                             const TcPlan &plan, const TcBuffers &buf, cudaStream_t stream,
                             bool *encoded)
 {
-    CUtensorMap tmK, tmQ;
+    CUtensorMap tmK, tmQ, tmKm;
+    memset(&tmKm, 0, sizeof tmKm);
+    const bool merged = K.bt && tc::encode_k_merged_map(&tmKm, K, g.L, g.Hkv, g.d);
     *encoded = tc::encode_k_map(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d) &&
                tc::encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.m, g.d, g.m, plan.gsub);
     if (!*encoded)
@@ -1161,6 +1199,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     TcArgs a;
     a.g = g;
     a.kp = tc::k_paging(K, g.n);
+    a.kp.merged = merged ? 1 : 0;
     a.rows = plan.rows;
     a.nrb = plan.nrb;
     a.gsub = plan.gsub;
@@ -1200,7 +1239,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
 
     // The traced build covers whole, contiguous units only; row blocks and paged caches run
     // untraced.
-    void (*kernel)(const CUtensorMap, const CUtensorMap, const TcArgs) =
+    void (*kernel)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const TcArgs) =
         K.bt ? (plan.nrb > 1 ? score_tc_kernel<false, true, true>
                              : score_tc_kernel<false, false, true>)
              : (plan.nrb > 1 ? score_tc_kernel<false, true, false>
@@ -1220,7 +1259,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kernel, tmK, tmQ, a);
+    return cudaLaunchKernelEx(&cfg, kernel, tmK, tmQ, tmKm, a);
 }
 
 }  // namespace dge

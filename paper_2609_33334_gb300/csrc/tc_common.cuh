@@ -93,6 +93,10 @@ __device__ __forceinline__ void transpose_sum16(float (&a)[16], int lane)
 struct KPaging {
     const int32_t *bt;   // block table [b][pps]
     int page_size, pps, num_pages, n;
+    int ps_shift;        // log2(page_size) for pages of 16, 32 or 64 slots
+    // The pool's slots run on across pages (page stride = page_size * slot stride): a tile
+    // whose pages are consecutive in the pool is one box of the merged map.
+    int merged;
 };
 
 // Largest number of pages a 128-key tile spans (page sizes 16, 32, 64 or multiples of 128).
@@ -103,20 +107,48 @@ constexpr int kPageWindowTiles = 32;
 constexpr int kPageWindow = kPageWindowTiles * kMaxTilePages;
 
 // The page ids of positions [k0, min(k0 + tiles * 128, n)) of sequence bb (tiles <=
-// kPageWindowTiles) into shared memory with 4-byte asynchronous copies, waited for before
-// returning (one round trip a window); ids[i] belongs to page k0 / page_size + i.  Invalid
-// ids are clamped when read.
-__device__ __forceinline__ void fetch_pages(int *ids, const KPaging &pg, int bb, int k0,
-                                            int tiles = kPageWindowTiles)
+// kPageWindowTiles) into shared memory (`buf`, 16-byte aligned, kPageWindow + 4 ints) with
+// asynchronous copies -- 16 bytes at a time where the table allows, 4 at its unaligned edges,
+// never past the entries needed.  fetch_pages_issue only issues them (fetch_pages_wait waits
+// for them); fetch_pages does both (one round trip a window).  Returns `ids`, with ids[i] the
+// id of page k0 / page_size + i.  Invalid ids are clamped when read.
+__device__ __forceinline__ const int *fetch_pages_issue(int *buf, const KPaging &pg, int bb,
+                                                        int k0, int tiles = kPageWindowTiles)
 {
     const int end = min(k0 + tiles * 128, pg.n);
-    const int p0 = k0 / pg.page_size, p1 = (end - 1) / pg.page_size;
-    const int32_t *src = pg.bt + (int64_t)bb * pg.pps;
-    for (int p = p0; p <= p1; ++p)
-        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_addr(ids + (p - p0))),
-                     "l"(src + p)
+    const int p0 = k0 / pg.page_size;
+    const int count = (end - 1) / pg.page_size - p0 + 1;
+    const int32_t *src = pg.bt + (int64_t)bb * pg.pps + p0;
+    // The same offset within 16 bytes on both sides, so the middle moves in 16-byte pieces.
+    int *ids = buf + (int)(((uintptr_t)src >> 2) & 3);
+    int i = 0;
+    for (; i < count && (((uintptr_t)(src + i)) & 15); ++i)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_addr(ids + i)),
+                     "l"(src + i)
                      : "memory");
+    for (; i + 4 <= count; i += 4)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(ptx::smem_addr(ids + i)),
+                     "l"(src + i)
+                     : "memory");
+    for (; i < count; ++i)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_addr(ids + i)),
+                     "l"(src + i)
+                     : "memory");
+    return ids;
+}
+
+// Waits for every page-id copy this thread has issued.
+__device__ __forceinline__ void fetch_pages_wait()
+{
     asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+__device__ __forceinline__ const int *fetch_pages(int *buf, const KPaging &pg, int bb, int k0,
+                                                  int tiles = kPageWindowTiles)
+{
+    const int *ids = fetch_pages_issue(buf, pg, bb, k0, tiles);
+    fetch_pages_wait();
+    return ids;
 }
 
 // One 128-key tile of K (nslab slabs of 64 columns, slab_bytes apart) into shared memory with
@@ -126,28 +158,53 @@ __device__ __forceinline__ void fetch_pages(int *ids, const KPaging &pg, int bb,
 // Positions past the cache read page 0, whose rows the callers mask.
 template <bool kPaged>
 __device__ __forceinline__ void load_k_tile(uint8_t *dst, uint32_t slab_bytes, int nslab,
-                                            const CUtensorMap *map, uint64_t *bar, int k0, int l,
-                                            int bb, int h, const KPaging &pg, const int *ids,
-                                            int w0, uint64_t policy)
+                                            const CUtensorMap *map, const CUtensorMap *merged,
+                                            uint64_t *bar, int k0, int l, int bb, int h,
+                                            const KPaging &pg, const int *ids, int w0,
+                                            uint64_t policy)
 {
     if constexpr (!kPaged) {
         for (int s = 0; s < nslab; ++s)
             ptx::tma_load_5d_hint(dst + s * slab_bytes, map, bar, s * 64, k0, h, bb, l, policy);
+    } else if (pg.page_size >= 128) {
+        // One page holds the whole tile.
+        int page = 0, slot = 0;
+        if (k0 < pg.n) {
+            const int pi = k0 / pg.page_size;
+            const int pid = ids[pi - w0 / pg.page_size];
+            page = (unsigned)pid < (unsigned)pg.num_pages ? pid : 0;
+            slot = k0 - pi * pg.page_size;
+        }
+        for (int s = 0; s < nslab; ++s)
+            ptx::tma_load_5d_hint(dst + s * slab_bytes, map, bar, s * 64, h, slot, page, l,
+                                  policy);
     } else {
-        const int rows = pg.page_size < 128 ? pg.page_size : 128;
-        const int npg = 128 / rows;
-        const int pbase = w0 / pg.page_size;
+        // 2..8 pages of 16, 32 or 64 slots; the tile and the window start on page boundaries.
+        const int npg = 128 >> pg.ps_shift;
+        const int i0 = (k0 - w0) >> pg.ps_shift;                            // first page in ids
+        const int valid = (pg.n - k0 + pg.page_size - 1) >> pg.ps_shift;    // pages before n
+        if (pg.merged && valid >= npg) {
+            // Pages handed out in order: the tile's pages follow each other in the pool.
+            const int first = ids[i0];
+            bool run = (unsigned)first <= (unsigned)(pg.num_pages - npg);
+            for (int j = 1; j < npg; ++j)
+                run = run && ids[i0 + j] == first + j;
+            if (run) {
+                for (int s = 0; s < nslab; ++s)
+                    ptx::tma_load_5d_hint(dst + s * slab_bytes, merged, bar, s * 64, h,
+                                          first << pg.ps_shift, l, 0, policy);
+                return;
+            }
+        }
         for (int j = 0; j < npg; ++j) {
-            const int pos = k0 + j * rows;
-            int page = 0, slot = 0;
-            if (pos < pg.n) {
-                const int pid = ids[pos / pg.page_size - pbase];
-                page = (pid >= 0 && pid < pg.num_pages) ? pid : 0;
-                slot = pos % pg.page_size;
+            int page = 0;
+            if (j < valid) {
+                const int pid = ids[i0 + j];
+                page = (unsigned)pid < (unsigned)pg.num_pages ? pid : 0;
             }
             for (int s = 0; s < nslab; ++s)
-                ptx::tma_load_5d_hint(dst + s * slab_bytes + j * rows * 128, map, bar, s * 64, h,
-                                      slot, page, l, policy);
+                ptx::tma_load_5d_hint(dst + s * slab_bytes + (j << pg.ps_shift) * 128, map, bar,
+                                      s * 64, h, 0, page, l, policy);
         }
     }
 }
@@ -158,8 +215,11 @@ __device__ __forceinline__ void load_k_tile(uint8_t *dst, uint32_t slab_bytes, i
 bool encode_5d(CUtensorMap *map, const TensorDesc &t, int L, int b, int heads, int rows, int d,
                int box_rows, int box_heads);
 bool have_tensor_maps();
-// Host: the K map of load_k_tile -- contiguous, or over a paged cache's pools (t.bt set).
+// Host: the K maps of load_k_tile -- contiguous, or over a paged cache's pools (t.bt set);
+// `merged` (paged caches) views the pool's slots as one run per layer, when the layout allows
+// it (KPaging::merged, from k_paging).
 bool encode_k_map(CUtensorMap *map, const TensorDesc &t, int L, int b, int Hkv, int n, int d);
+bool encode_k_merged_map(CUtensorMap *map, const TensorDesc &t, int L, int Hkv, int d);
 KPaging k_paging(const TensorDesc &t, int n);
 
 }  // namespace tc

@@ -210,20 +210,33 @@ def bf16_bits(t: torch.Tensor) -> np.ndarray:
 
 
 def paged_layout(cache: torch.Tensor, page_size: int, seed: int = 0, spare_pages: int = 3,
-                 extra_table_pages: int = 1, head_major: bool = False) -> tuple:
+                 extra_table_pages: int = 1, head_major: bool = False,
+                 order: str = "random") -> tuple:
     """Lay a contiguous cache [L][b][Hkv][n][d] out as a paged one, the way a paged-attention
-    server keeps it: returns (pool [L][num_pages][page_size][Hkv][d], or with ``head_major``
-    [L][num_pages][Hkv][page_size][d], and block_table int32 [b][pages_per_seq]).  Sequences get pages in a seeded random order (shared by all
-    layers), the pool has ``spare_pages`` pages no sequence uses, and the table has
-    ``extra_table_pages`` entries per sequence past the cache (set to -1).  Every slot that
-    holds no cache position is NaN, so a read of one shows in the results.  Pure layout: no
-    arithmetic of the method."""
+    server keeps it: returns the pool [L][num_pages][page_size][Hkv][d] (``head_major``:
+    [L][num_pages][Hkv][page_size][d]) and the block table, int32 [b][pages_per_seq].
+    Sequences get pages in a seeded random order shared by all layers (``order=
+    "sequential"``: each sequence's pages one after another, as a fresh allocator hands them
+    out; ``"runs"``: sequential with one page in eight swapped with a random other).  The pool
+    has ``spare_pages`` pages no sequence uses, and the table ``extra_table_pages`` entries per
+    sequence past the cache (set to -1).  Every slot that holds no cache position is NaN, so a
+    read of one shows in the results.  Pure layout: no arithmetic of the method."""
     L, b, Hkv, n, d = cache.shape
     used = (n + page_size - 1) // page_size
     pps = used + extra_table_pages
     num_pages = b * used + spare_pages
     rng = np.random.default_rng(seed)
-    perm = rng.permutation(num_pages)[:b * used].reshape(b, used)
+    if order == "random":
+        flat = rng.permutation(num_pages)
+    else:
+        flat = np.arange(num_pages)
+        if order == "runs":
+            for i in rng.choice(num_pages, num_pages // 8, replace=False):
+                j = rng.integers(num_pages)
+                flat[i], flat[j] = flat[j], flat[i]
+        elif order != "sequential":
+            raise ValueError(order)
+    perm = flat[:b * used].reshape(b, used)
     table = np.full((b, pps), -1, dtype=np.int32)
     table[:, :used] = perm
     shape = (L, num_pages, Hkv, page_size, d) if head_major else (L, num_pages, page_size, Hkv, d)

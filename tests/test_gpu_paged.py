@@ -33,9 +33,11 @@ def built():
     _build.build()
 
 
-def _paged(tens, page_size, seed=0, head_major=False):
-    K, bt = inputs.paged_layout(tens["K"], page_size, seed=seed, head_major=head_major)
-    V, bt2 = inputs.paged_layout(tens["V"], page_size, seed=seed, head_major=head_major)
+def _paged(tens, page_size, seed=0, head_major=False, order="random"):
+    K, bt = inputs.paged_layout(tens["K"], page_size, seed=seed, head_major=head_major,
+                                order=order)
+    V, bt2 = inputs.paged_layout(tens["V"], page_size, seed=seed, head_major=head_major,
+                                 order=order)
     assert torch.equal(bt, bt2)
     return K, V, api.Paging(block_table=bt, page_size=page_size, head_major=head_major)
 
@@ -184,3 +186,21 @@ def test_head_major_pages(name, page_size):
             for h in range(wl.Hkv):
                 assert torch.equal(Kn[l, b, h, :B], ref["Kc"][offs[u]:offs[u] + B])
                 u += 1
+
+
+@pytest.mark.parametrize("order", ["sequential", "runs"])
+@pytest.mark.parametrize("page_size", [16, 64])
+@pytest.mark.parametrize("name", ["c2_small", "c5_small", "c4_small"])
+def test_consecutive_pages(name, page_size, order):
+    """Pages handed out in order (and in order with some swapped): tiles whose pages follow
+    each other in the pool load as one box of the merged map, the others page by page; the
+    outputs are the contiguous run's either way."""
+    wl = CASES[name]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    ref = api.evict(p, tens["K"], tens["V"], tens["Q"], want_scores=True)
+    K, V, pg = _paged(tens, page_size, seed=7, order=order)
+    got = api.evict(p, K, V, tens["Q"], want_scores=True, paging=pg)
+    torch.cuda.synchronize()
+    for k in ("idx", "Kc", "Vc", "scores"):
+        assert torch.equal(got[k], ref[k]), k
