@@ -181,7 +181,6 @@ struct Smem {
     float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
     float *xch;          // [kAccBufs][kEpiWG][128] phase-2 partial column sums
-    int *xcnt;           // [kAccBufs][4] arrivals (row-block path: exactly one finaliser)
     int *pages;          // [tc::kPageWindow + 4] page ids of the producer's window (paged caches)
 };
 
@@ -193,7 +192,7 @@ __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
            + kStageBytes                          // lse merge staging
            + kCtrlBytes                           // barriers, tmem holder, flags
            + (2 * 256 + 2 * kEpiWG * 4 * kMaxGroups * 16) * 4 + 16
-           + kAccBufs * kEpiWG * kTile * 4 + kAccBufs * 4 * 4 + (tc::kPageWindow + 4) * 4;
+           + kAccBufs * kEpiWG * kTile * 4 + (tc::kPageWindow + 4) * 4;
 }
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
@@ -222,8 +221,6 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int ks
     off += 16;
     s.xch = reinterpret_cast<float *>(raw + off);
     off += kAccBufs * kEpiWG * kTile * 4;
-    s.xcnt = reinterpret_cast<int *>(raw + off);
-    off += kAccBufs * 4 * 4;
     s.pages = reinterpret_cast<int *>(raw + off);
     return s;
 }
@@ -361,10 +358,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         flag[kFlagSArm] = -1;
         // Phase-2 exchange: one barrier per accumulator and lane quarter, one arrival per
         // warpgroup.
-        for (int i = 0; i < kAccBufs * 4; ++i) {
+        for (int i = 0; i < kAccBufs * 4; ++i)
             ptx::mbar_init(&sm.bar[kBarXch + i], kEpiWG);
-            sm.xcnt[i] = 0;
-        }
         ptx::fence_mbar_init();
     }
     // Query rows R .. r_pad-1 are never written by TMA: zero them once so the padded
@@ -908,6 +903,19 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         // rewritten only after accumulator ab is refilled, which needs every
                         // warp's release below, the last warp's after its reads.
                         const long long cx = tclock<kTr>();
+                        if constexpr (kFx) {
+                            // Row blocks add into the unit's score row in integers (2^-40
+                            // units), so every warpgroup adds its own partial sum: the order of
+                            // the additions does not matter and no warp waits for another.
+                            // The scaling by 2^40 is exact in fp32, so this is a rounding of
+                            // the exact product.
+                            if (task_ok && key < T.k_hi)
+                                atomicAdd(fx_row + key, (unsigned long long)__float2ll_rn(
+                                                            (acc.x + acc.y) * 0x1p40f));
+                            cy_xch += tclock<kTr>() - cx;
+                            release_acc(ab, 1u);
+                            continue;
+                        }
                         float *xs = sm.xch + ab * kEpiWG * kTile;
                         xs[wg * kTile + kl] = acc.x + acc.y;
                         __syncwarp();
@@ -916,18 +924,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         // both find it so: they store the same value).
                         int last = 0;
                         if (lane == 0) {
-                            if (kFx) {
-                                // Row blocks add their sums atomically, so exactly one warp may
-                                // finalise: the one whose count completes the three arrivals.
-                                __threadfence_block();
-                                last = atomicAdd(&sm.xcnt[ab * 4 + quarter], 1) % kEpiWG ==
-                                       kEpiWG - 1;
-                                __threadfence_block();
-                            } else {
-                                uint64_t *xb = &sm.bar[kBarXch + ab * 4 + quarter];
-                                last = ptx::mbar_test_token(xb, ptx::mbar_arrive_token(xb)) ? 1
-                                                                                           : 0;
-                            }
+                            uint64_t *xb = &sm.bar[kBarXch + ab * 4 + quarter];
+                            last = ptx::mbar_test_token(xb, ptx::mbar_arrive_token(xb)) ? 1 : 0;
                         }
                         last = __shfl_sync(0xffffffffu, last, 0);
                         __syncwarp();  // lane 0's acquire orders the other lanes' reads
@@ -936,16 +934,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
 #pragma unroll
                             for (int w = 1; w < kEpiWG; ++w)
                                 total += xs[w * kTile + kl];
-                            if (task_ok && key < T.k_hi) {
-                                // Row blocks of one unit add up exactly in integers; the scaling
-                                // by 2^40 is exact in fp32, so this matches a rounding of the
-                                // exact product.
-                                if (kFx)
-                                    atomicAdd(fx_row + key,
-                                              (unsigned long long)__float2ll_rn(total * 0x1p40f));
-                                else
-                                    raw_row[key] = total;
-                            }
+                            if (task_ok && key < T.k_hi)
+                                raw_row[key] = total;
                         }
                         cy_xch += tclock<kTr>() - cx;
                         release_acc(ab, 1u);
