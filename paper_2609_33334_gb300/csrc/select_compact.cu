@@ -99,6 +99,7 @@ __device__ __forceinline__ void scan_warp_counts(const int *cnt, int *base)
 
 constexpr int kRadixBits = 11;
 constexpr int kRadixBins = 1 << kRadixBits;
+static_assert(kRadixBins == 2 * kSelThreads, "two bins per thread in the bin search");
 
 // Shared-memory scratch of the selection helpers.
 struct SelScratch {
@@ -116,15 +117,16 @@ struct SelScratch {
 // serialise.  Called by every thread of a block of kSelThreads.
 template <typename KeyAt>
 __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, uint32_t &T,
-                                int &need_eq)
+                                int &need_eq, uint32_t kmin = 0xffffffffu, uint32_t kmax = 0u,
+                                bool have_range = false)
 {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    uint32_t kmin = 0xffffffffu, kmax = 0u;
-    for (int j = tid; j < C; j += kSelThreads) {
-        const uint32_t k = key_at(j);
-        kmin = min(kmin, k);
-        kmax = max(kmax, k);
-    }
+    if (!have_range)
+        for (int j = tid; j < C; j += kSelThreads) {
+            const uint32_t k = key_at(j);
+            kmin = min(kmin, k);
+            kmax = max(kmax, k);
+        }
     kmin = __reduce_min_sync(0xffffffffu, kmin);
     kmax = __reduce_max_sync(0xffffffffu, kmax);
     if (lane == 0) {
@@ -163,14 +165,12 @@ __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, u
                 atomicAdd(&sc.hist[(k >> shift) & bmask], 1u);
         }
         __syncthreads();
-        if (warp == 0) {
-            // Suffix counts over the bins, from the top: a lane sums kRadixBins / 32
-            // consecutive bins (bins above bmask are empty).
-            constexpr int per = kRadixBins / 32;
-            const int tb = kRadixBins - 1 - lane * per;   // this lane's bins: tb, tb-1, ...
-            uint32_t local = 0;
-            for (int q = 0; q < per; ++q)
-                local += sc.hist[tb - q];
+        {
+            // Counts from the top bin down: thread t holds bins tb and tb - 1, tb = top - 2t
+            // (bins above bmask are empty); a block scan gives the count above each pair.
+            const int tb = kRadixBins - 1 - 2 * tid;
+            const uint32_t c_hi = sc.hist[tb], c_lo = sc.hist[tb - 1];
+            const uint32_t local = c_hi + c_lo;
             uint32_t incl = local;
 #pragma unroll
             for (int off = 1; off < 32; off <<= 1) {
@@ -178,24 +178,32 @@ __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, u
                 if (lane >= off)
                     incl += o;
             }
-            uint32_t run = incl - local;
-            if (run < (uint32_t)rank && run + local >= (uint32_t)rank) {
-                for (int q = 0; q < per; ++q) {
-                    const uint32_t c = sc.hist[tb - q];
-                    if (run + c >= (uint32_t)rank) {
-                        sc.prefix = prefix | ((uint32_t)(tb - q) << shift);
-                        sc.rank = rank - (int)run;
-                        break;
-                    }
-                    run += c;
+            if (lane == 31)
+                sc.warp_a[warp] = (int)incl;
+            __syncthreads();
+            if (warp == 0) {
+                const uint32_t v = (uint32_t)sc.warp_a[lane];
+                uint32_t wi = v;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const uint32_t o = __shfl_up_sync(0xffffffffu, wi, off);
+                    if (lane >= off)
+                        wi += o;
                 }
+                sc.warp_b[lane] = (int)(wi - v);
+            }
+            __syncthreads();
+            const uint32_t run = (uint32_t)sc.warp_b[warp] + incl - local;
+            if (run < (uint32_t)rank && run + local >= (uint32_t)rank) {
+                const bool hi_bin = run + c_hi >= (uint32_t)rank;
+                sc.prefix = prefix | ((uint32_t)(hi_bin ? tb : tb - 1) << shift);
+                sc.rank = rank - (int)(hi_bin ? run : run + c_hi);
             }
         }
         __syncthreads();
         prefix = sc.prefix;
         rank = sc.rank;
         mask |= bmask << shift;
-        __syncthreads();
     }
     T = npass == 0 ? kmax : prefix;   // npass == 0: every key is equal
     need_eq = rank;
@@ -252,6 +260,78 @@ __device__ void ordered_compaction(KeyAt key_at, int C, uint32_t T, int need_eq,
     }
 }
 
+// Block-wide exclusive scan of one value per thread (thread order); every thread of a block
+// of kSelThreads calls it.  Returns the sum over lower threads; *total (nullable) = the sum.
+__device__ __forceinline__ int block_exclusive_scan(int v, SelScratch &sc, int *total = nullptr)
+{
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    int incl = v;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int o = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off)
+            incl += o;
+    }
+    if (lane == 31)
+        sc.warp_a[warp] = incl;
+    __syncthreads();
+    const int wv = lane < kSelWarps ? sc.warp_a[lane] : 0;
+    int wi = wv;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int o = __shfl_up_sync(0xffffffffu, wi, off);
+        if (lane >= off)
+            wi += o;
+    }
+    const int before = __shfl_sync(0xffffffffu, wi - wv, warp);
+    if (total)
+        *total = __shfl_sync(0xffffffffu, wi, 31);
+    __syncthreads();   // warp_a is free again
+    return before + incl - v;
+}
+
+// ordered_compaction for C <= 32 * kSelThreads in one pass over the keys: warp w's range is
+// cut into 32-key segments, and a ballot per segment hands lane s the masks of segment s (keys
+// above T, keys equal to T).  Two block scans give each lane its share of the equal keys and
+// its first output slot; it then writes its kept positions in order.
+template <typename KeyAt>
+__device__ void ordered_compaction_masks(KeyAt key_at, int C, uint32_t T, int need_eq, int keep,
+                                         int s0, int32_t *out, SelScratch &sc)
+{
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int per_w = ((C + kSelWarps - 1) / kSelWarps + 31) & ~31;   // <= 1024
+    const int w_lo = min(C, warp * per_w), w_hi = min(C, w_lo + per_w);
+    uint32_t gtm = 0, eqm = 0;
+    for (int q = 0; q < per_w / 32; ++q) {
+        const int j = w_lo + 32 * q + lane;
+        const uint32_t k = j < w_hi ? key_at(j) : 0u;
+        const uint32_t gb = __ballot_sync(0xffffffffu, j < w_hi && k > T);
+        const uint32_t eb = __ballot_sync(0xffffffffu, j < w_hi && k == T);
+        if (lane == q) {
+            gtm = gb;
+            eqm = eb;
+        }
+    }
+    // Equal keys before this segment; this lane keeps the lowest of its own up to need_eq.
+    const int eq_before = block_exclusive_scan(__popc(eqm), sc);
+    int take = min(__popc(eqm), max(0, need_eq - eq_before));
+    uint32_t sel = gtm;
+    for (uint32_t e = eqm; take > 0; --take) {
+        const uint32_t low = e & (0u - e);
+        sel |= low;
+        e ^= low;
+    }
+    int pos = block_exclusive_scan(__popc(sel), sc);
+    const int seg0 = s0 + w_lo + 32 * lane;
+    while (sel) {
+        const int b = __ffs(sel) - 1;
+        if (pos < keep)
+            out[pos] = seg0 + b;
+        ++pos;
+        sel &= sel - 1;
+    }
+}
+
 template <bool SMEM>
 __global__ void __launch_bounds__(kSelThreads)
 select_kernel(const float *__restrict__ scores, int32_t *__restrict__ idx, SelectParams p)
@@ -290,7 +370,10 @@ select_kernel(const float *__restrict__ scores, int32_t *__restrict__ idx, Selec
     uint32_t T;
     int need_eq;
     radix_threshold(key_at, C, keep, scr, T, need_eq);
-    ordered_compaction(key_at, C, T, need_eq, keep, s0, out + s0, scr);
+    if (C <= 32 * kSelThreads)
+        ordered_compaction_masks(key_at, C, T, need_eq, keep, s0, out + s0, scr);
+    else
+        ordered_compaction(key_at, C, T, need_eq, keep, s0, out + s0, scr);
 }
 
 cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const float *scores,
@@ -319,15 +402,17 @@ cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const flo
 // Pooling and selection fused (the evict path, P <= kPsMaxP): one CTA per unit loads the
 // unit's raw scores into shared memory once, pools them (the same arithmetic and order as
 // pool_kernel, so the pooled values are bit-identical), optionally writes them out, and
-// selects from the shared-memory copy.  The kernel is bound by instruction issue, so the
-// radix select takes three passes (11, 11 and 10 bits) and the position-ordered compaction
-// two: a warp's count of kept candidates follows from its counts of keys above and equal to
-// the threshold and the equal keys before it.
+// selects from the shared-memory copy.  The kernel is latency- and issue-bound (one CTA per
+// SM, block barriers between its steps): pooling reads each score once from shared memory (a
+// 16-byte load gives a lane four consecutive positions, the neighbours come by shuffles; R
+// guard cells of the pool's neutral value on each side of the row leave every window sum or
+// max bit-identical to the clipped one), the key range comes with the key write, the radix
+// select's bin search is a block scan, and the position-ordered compaction reads the keys
+// once.
 
 constexpr int kPsThreads = 1024;
 constexpr int kPsPer = 32;                       // positions pooled per thread (registers)
 constexpr int kPsMaxP = kPsThreads * kPsPer;     // 32768
-
 
 // Pooled value at position j of a row of P raw scores in shared memory.  R > 0: the pool
 // radius known at compile time (interior positions unrolled); R < 0: radius r at run time.
@@ -350,12 +435,15 @@ __device__ __forceinline__ float pool_at(const float *sraw, int j, int P, int r,
     return POOL == DGE_POOL_AVG ? x * (1.0f / (float)kernel) : x;
 }
 
+constexpr int kPsGuard = 4;                      // guard cells on each side of the row
+
 template <int POOL, int R>
 __global__ void __launch_bounds__(kPsThreads, 1)
 pool_select_kernel(const float *__restrict__ raw, float *__restrict__ pooled_out,
                    int32_t *__restrict__ idx, SelectParams p, int kernel)
 {
-    extern __shared__ __align__(16) uint32_t sbuf[];  // [P]: raw scores, then pooled keys
+    // [guard][P rounded up to 128][guard]: raw scores, then pooled keys in place
+    extern __shared__ __align__(16) uint32_t sbuf[];
     __shared__ SelScratch sc;
 
     const int tid = threadIdx.x;
@@ -369,26 +457,99 @@ pool_select_kernel(const float *__restrict__ raw, float *__restrict__ pooled_out
 
     // Raw scores to shared memory, pooled values to registers, then keys in place.
     const float *row = raw + u * (int64_t)P;
-    float *sraw = reinterpret_cast<float *>(sbuf);
+    uint32_t *skey = sbuf + kPsGuard;
+    float *sraw = reinterpret_cast<float *>(skey);
     for (int j = tid; j < P; j += kPsThreads)
         sraw[j] = row[j];
+    if (tid < kPsGuard) {
+        const float neutral = POOL == DGE_POOL_MAX ? -INFINITY : 0.f;
+        sraw[-1 - tid] = neutral;
+        sraw[P + tid] = neutral;
+    }
     __syncthreads();
+    // Position of value i of this thread: chunks of 128 positions, chunk c to warp c % 32;
+    // a lane holds 4 consecutive positions of each of its chunks (compile-time radius), or
+    // positions tid + 1024 i (run-time radius).
+    constexpr bool kChunked = R >= 0 && R <= kPsGuard;
+    const int lane = tid & 31, warp = tid >> 5;
+    auto pos_of = [&](int i) {
+        return kChunked ? 128 * (warp + 32 * (i >> 2)) + 4 * lane + (i & 3) : tid + i * kPsThreads;
+    };
     float v[kPsPer];
+    if constexpr (kChunked) {
+        constexpr int RR = R > 0 ? R : 0;
 #pragma unroll
-    for (int i = 0; i < kPsPer; ++i) {
-        const int j = tid + i * kPsThreads;
-        v[i] = j < P ? pool_at<POOL, R>(sraw, j, P, kernel / 2, kernel) : 0.f;
+        for (int c = 0; c < kPsPer / 4; ++c) {
+            const int base = 128 * (warp + 32 * c);
+            if (base < P) {   // warp-uniform
+                const float4 a = *reinterpret_cast<const float4 *>(sraw + base + 4 * lane);
+                // w[4 + t] = position 4 * lane + t of the chunk, t = -4 .. 7.
+                float w[12];
+                w[4] = a.x;
+                w[5] = a.y;
+                w[6] = a.z;
+                w[7] = a.w;
+#pragma unroll
+                for (int t = 1; t <= RR; ++t) {
+                    const float left = __shfl_up_sync(0xffffffffu, w[8 - t], 1);
+                    const float right = __shfl_down_sync(0xffffffffu, w[3 + t], 1);
+                    w[4 - t] = lane == 0 ? sraw[base - t] : left;
+                    w[7 + t] = lane == 31 ? sraw[base + 127 + t] : right;
+                }
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                    if (POOL == DGE_POOL_NONE) {
+                        v[4 * c + t] = w[4 + t];
+                        continue;
+                    }
+                    float x = POOL == DGE_POOL_MAX ? -INFINITY : 0.f;
+#pragma unroll
+                    for (int q = -RR; q <= RR; ++q)
+                        x = POOL == DGE_POOL_MAX ? fmaxf(x, w[4 + t + q]) : x + w[4 + t + q];
+                    v[4 * c + t] = POOL == DGE_POOL_AVG ? x * (1.0f / (float)(2 * RR + 1)) : x;
+                }
+            } else {
+#pragma unroll
+                for (int t = 0; t < 4; ++t)
+                    v[4 * c + t] = 0.f;
+            }
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < kPsPer; ++i) {
+            const int j = tid + i * kPsThreads;
+            v[i] = j < P ? pool_at<POOL, R>(sraw, j, P, kernel / 2, kernel) : 0.f;
+        }
     }
     __syncthreads();
     float *pout = pooled_out ? pooled_out + u * (int64_t)P : nullptr;
+    uint32_t kmin = 0xffffffffu, kmax = 0u;   // range of the candidate keys [s0, P)
+    uint32_t kv[kPsPer];
 #pragma unroll
     for (int i = 0; i < kPsPer; ++i) {
-        const int j = tid + i * kPsThreads;
+        const int j = pos_of(i);
+        kv[i] = float_key(v[i]);
         if (j < P) {
             if (pout)
                 pout[j] = v[i];
-            sbuf[j] = float_key(v[i]);
+            if (j >= s0) {
+                kmin = min(kmin, kv[i]);
+                kmax = max(kmax, kv[i]);
+            }
         }
+    }
+    if constexpr (kChunked) {
+        // Four consecutive keys at once (positions past P land in the chunk padding).
+#pragma unroll
+        for (int c = 0; c < kPsPer / 4; ++c)
+            if (pos_of(4 * c) < P)
+                *reinterpret_cast<uint4 *>(skey + pos_of(4 * c)) =
+                    make_uint4(kv[4 * c], kv[4 * c + 1], kv[4 * c + 2], kv[4 * c + 3]);
+    } else {
+#pragma unroll
+        for (int i = 0; i < kPsPer; ++i)
+            if (pos_of(i) < P)
+                skey[pos_of(i)] = kv[i];
     }
     __syncthreads();
 
@@ -403,12 +564,12 @@ pool_select_kernel(const float *__restrict__ raw, float *__restrict__ pooled_out
             out[s0 + j] = s0 + j;
         return;
     }
-    const uint32_t *keys = sbuf + s0;
+    const uint32_t *keys = skey + s0;
     auto key_at = [&](int j) -> uint32_t { return keys[j]; };
     uint32_t T;
     int need_eq;
-    radix_threshold(key_at, C, keep, sc, T, need_eq);
-    ordered_compaction(key_at, C, T, need_eq, keep, s0, out + s0, sc);
+    radix_threshold(key_at, C, keep, sc, T, need_eq, kmin, kmax, true);
+    ordered_compaction_masks(key_at, C, T, need_eq, keep, s0, out + s0, sc);
 }
 
 bool pool_select_supported(const Geometry &g) { return g.P <= kPsMaxP; }
@@ -419,7 +580,8 @@ cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, cons
     SelectParams p;
     p.g = g;
     p.layers = layers;
-    const size_t smem = (size_t)max(g.P, 1) * sizeof(uint32_t);
+    // The row rounded up to whole 128-position chunks, with guard cells on both sides.
+    const size_t smem = (size_t)(((max(g.P, 1) + 127) & ~127) + 2 * kPsGuard) * sizeof(uint32_t);
     using KernT = void (*)(const float *, float *, int32_t *, SelectParams, int);
     KernT kern;
     if (g.pool == DGE_POOL_MAX)
