@@ -121,7 +121,7 @@ struct Plan {
     int nchunks = 0;
     TcPlan tc = {};          // tensor-core path decomposition (SCORED only)
     size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, off_count = 0,
-           off_ready = 0, off_rawfx = 0, off_unitflag = 0, ws_bytes = 0;
+           off_ready = 0, off_rawfx = 0, off_unitflag = 0, off_units = 0, ws_bytes = 0;
 };
 
 constexpr int kScoredChunkKeys = 2048;
@@ -252,6 +252,9 @@ int make_plan(const dge_problem *p, Plan &plan)
         off = align256(off + (size_t)g.U * nrb * sizeof(uint32_t));
         plan.off_ready = off;
         off = align256(off + (size_t)g.U * nrb * sizeof(uint32_t));
+        // Units left for the recompute: count, then ids.
+        plan.off_units = off;
+        off = align256(off + (size_t)(g.U + 1) * sizeof(uint32_t));
         if (nrb > 1) {
             // Row blocks of one unit add their column sums in fixed point (exact, so the
             // order of the additions does not matter), and their range flags per unit.
@@ -379,13 +382,20 @@ int run_h2o_tc(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void 
     *done = true;
     if (supplied)
         return DGE_OK;
+    // Every row of every unit is a query row here, so the per-unit grids are large: the
+    // recompute runs over a device-side list of the flagged units (usually empty).
+    UnitSel units;
+    units.sel = ws_at<uint32_t>(ws, plan.off_units);
+    units.list = true;
+    DGE_LAUNCH("recompute_list", stream,
+               launch_collect_units(ready, g.U, ws_at<uint32_t>(ws, plan.off_units), stream));
     DGE_LAUNCH("recompute_lse", stream,
                launch_lse_partial(K, Q, g, plan.rows_per_block, plan.chunk_keys, partial, stream,
-                                  ready));
+                                  units));
     DGE_LAUNCH("recompute_combine", stream,
-               launch_combine_lse(partial, g.U * g.R, plan.nchunks, lse2, stream, ready, g.R));
+               launch_combine_lse(partial, g.U * g.R, plan.nchunks, lse2, stream, units, g.R));
     DGE_LAUNCH("recompute_colsum", stream,
-               launch_colsum_keys(K, Q, g, lse2, raw, stream, ready));
+               launch_colsum_keys(K, Q, g, lse2, raw, stream, units));
     if (lse_out)
         DGE_LAUNCH("lse_export", stream,
                    launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
@@ -479,13 +489,16 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
                            launch_unit_flags(ready, nrb, g.U, unit_flag, stream));
             }
             // Units whose row sums left fp32's safe range (flag 2) are recomputed with the
-            // running-maximum kernels; every other unit returns at once.
+            // running-maximum kernels; every other unit's CTA returns at once (one CTA per
+            // unit: cheaper than collecting a list first).
+            UnitSel units;
+            units.sel = unit_flag;
             DGE_LAUNCH("recompute_lse", stream,
-                       launch_lse_partial(K, Q, g, g.R, g.n, partial, stream, unit_flag));
+                       launch_lse_partial(K, Q, g, g.R, g.n, partial, stream, units));
             DGE_LAUNCH("recompute_combine", stream,
-                       launch_combine_lse(partial, g.U * g.R, 1, lse2, stream, unit_flag, g.R));
+                       launch_combine_lse(partial, g.U * g.R, 1, lse2, stream, units, g.R));
             DGE_LAUNCH("recompute_colsum", stream,
-                       launch_colsum_rows(K, Q, g, g.P, lse2, raw, stream, unit_flag));
+                       launch_colsum_rows(K, Q, g, g.P, lse2, raw, stream, units));
             if (lse_out)
                 DGE_LAUNCH("lse_export", stream,
                            launch_lse_export(tb.part, plan.tc.nchunks, plan.tc.r4, lse2,

@@ -5,18 +5,28 @@
 
 namespace dge {
 
-// Scoring on the warp-level tensor core path (score_mma.cu).  `only` (nullable, [U])
-// restricts the work to units whose entry equals kUnitRecompute.
+// Scoring on the warp-level tensor core path (score_mma.cu).  A UnitSel restricts the work:
+// sel == nullptr, every unit; list false, the units whose flag sel[u] equals kUnitRecompute;
+// list true, the units of a device-side list (sel[0] = count, sel[1 ..] = ids, as written by
+// launch_collect_units), taken by a capped grid, so that an empty list costs little however
+// many units there are.
 constexpr uint32_t kUnitRecompute = 2;
+struct UnitSel {
+    const uint32_t *sel = nullptr;
+    bool list = false;
+};
 cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int rows_per_block, int chunk_keys, float2 *partial,
-                               cudaStream_t stream, const uint32_t *only = nullptr);
+                               cudaStream_t stream, UnitSel units = {});
 cudaError_t launch_combine_lse(const float2 *partial, int64_t total_rows, int nchunks,
-                               float *lse2, cudaStream_t stream, const uint32_t *only = nullptr,
+                               float *lse2, cudaStream_t stream, UnitSel units = {},
                                int rows_per_unit = 1);
 cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int chunk_keys, const float *lse2, float *raw,
-                               cudaStream_t stream, const uint32_t *only = nullptr);
+                               cudaStream_t stream, UnitSel units = {});
+// The units whose flag (flags[U]) equals kUnitRecompute into units[1 + U] (count first).
+cudaError_t launch_collect_units(const uint32_t *flags, int64_t U, uint32_t *units,
+                                 cudaStream_t stream);
 
 // Scoring on the tcgen05 path (score_tc.cu).
 struct TcPlan {
@@ -48,7 +58,7 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
                             bool *encoded);
 cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                const float *lse2, float *raw, cudaStream_t stream,
-                               const uint32_t *only = nullptr);
+                               UnitSel units = {});
 
 // H2O scoring on the tcgen05 path (h2o_tc.cu): query blocks of pb positions x G heads.
 struct H2oPlan {

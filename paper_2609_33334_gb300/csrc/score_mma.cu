@@ -105,23 +105,44 @@ __device__ __forceinline__ int max_row_position(const Geometry &g, int r0, int r
     return g.n - 1;
 }
 
+// The units a launch covers (UnitSel): every unit, one CTA per block of work (sel ==
+// nullptr); the units whose flag sel[u] equals kUnitRecompute (the other CTAs return at
+// once); or the units of a list (units[0] = count, units[1 ..] = ids), whose blocks the CTAs
+// of a capped grid take in turn -- a launch for an empty list costs one read per CTA however
+// large the problem.  vblocks is the number of blocks of work, vblock_id the global block
+// index of the vb-th, vblock_skip whether a block of unit u has nothing to do.
+__device__ __forceinline__ int64_t vblocks(const UnitSel &us, int64_t U, int64_t per_unit)
+{
+    return (us.sel && us.list ? (int64_t)us.sel[0] : U) * per_unit;
+}
+__device__ __forceinline__ int64_t vblock_id(const UnitSel &us, int64_t per_unit, int64_t vb)
+{
+    return us.sel && us.list ? (int64_t)us.sel[1 + vb / per_unit] * per_unit + vb % per_unit
+                             : vb;
+}
+__device__ __forceinline__ bool vblock_skip(const UnitSel &us, int64_t u)
+{
+    return us.sel && !us.list && us.sel[u] != kUnitRecompute;
+}
+constexpr int64_t kListGrid = 1024;   // CTAs of a launch over a unit list
+__host__ inline int64_t grid_for(const UnitSel &us, int64_t blocks)
+{
+    return us.sel && us.list && blocks > kListGrid ? kListGrid : blocks;
+}
+
 // ---------------------------------------------------------------------------
 // Phase 1: per-row (max, sum) partials over one key chunk.
 // Block = (unit, row block, key chunk), flattened as ((u * nrb) + rb) * nchunks + chunk.
 // partial layout: [u][R][nchunks] float2 (max in base-2 units, sum of 2^{x - max}).
 template <int D, int MAX_NTW>
-__global__ void __launch_bounds__(kThreads)
-lse_partial_kernel(TensorDesc K, TensorDesc Q, Geometry g, int rows_per_block, int nrb,
-                   int chunk_keys, int nchunks, float2 *__restrict__ partial,
-                   const uint32_t *__restrict__ only)
+__device__ void lse_partial_block(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                                  int rows_per_block, int nrb, int chunk_keys, int nchunks,
+                                  float2 *__restrict__ partial, int64_t bid)
 {
     extern __shared__ __align__(16) uint8_t smem[];
-    const int64_t bid = blockIdx.x;
     const int chunk = (int)(bid % nchunks);
     const int rb = (int)((bid / nchunks) % nrb);
     const int64_t u = bid / ((int64_t)nchunks * nrb);
-    if (only && only[u] != kUnitRecompute)
-        return;
     int l, bb, h;
     unit_coords(g, u, l, bb, h);
     const int r0 = rb * rows_per_block;
@@ -220,41 +241,57 @@ lse_partial_kernel(TensorDesc K, TensorDesc Q, Geometry g, int rows_per_block, i
         }
 }
 
+template <int D, int MAX_NTW>
+__global__ void __launch_bounds__(kThreads)
+lse_partial_kernel(TensorDesc K, TensorDesc Q, Geometry g, int rows_per_block, int nrb,
+                   int chunk_keys, int nchunks, float2 *__restrict__ partial, UnitSel us)
+{
+    const int64_t per = (int64_t)nrb * nchunks;
+    const int64_t total = vblocks(us, g.U, per);
+    for (int64_t vb = blockIdx.x; vb < total; vb += gridDim.x) {
+        const int64_t bid = vblock_id(us, per, vb);
+        if (vblock_skip(us, bid / per))
+            continue;
+        lse_partial_block<D, MAX_NTW>(K, Q, g, rows_per_block, nrb, chunk_keys, nchunks, partial,
+                                      bid);
+        __syncthreads();   // shared memory is reused by the next block of work
+    }
+}
+
 // lse_r = M + log2(sum_c z_c 2^{m_c - M}) over the chunks of row r.
 __global__ void combine_lse_kernel(const float2 *__restrict__ partial, int64_t total_rows,
-                                   int nchunks, float *__restrict__ lse2,
-                                   const uint32_t *__restrict__ only, int rows_per_unit)
+                                   int nchunks, float *__restrict__ lse2, UnitSel us,
+                                   int rows_per_unit)
 {
-    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= total_rows)
-        return;
-    if (only && only[i / rows_per_unit] != kUnitRecompute)
-        return;
-    const float2 *p = partial + i * nchunks;
-    float M = neg_inf();
-    for (int c = 0; c < nchunks; ++c)
-        M = fmaxf(M, p[c].x);
-    float Z = 0.f;
-    for (int c = 0; c < nchunks; ++c)
-        Z += p[c].y * ex2(p[c].x - M);
-    lse2[i] = M + log2f(Z);
+    const int64_t total = us.sel && us.list ? (int64_t)us.sel[0] * rows_per_unit : total_rows;
+    for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < total;
+         v += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i = vblock_id(us, rows_per_unit, v);
+        if (vblock_skip(us, i / rows_per_unit))
+            continue;
+        const float2 *p = partial + i * nchunks;
+        float M = neg_inf();
+        for (int c = 0; c < nchunks; ++c)
+            M = fmaxf(M, p[c].x);
+        float Z = 0.f;
+        for (int c = 0; c < nchunks; ++c)
+            Z += p[c].y * ex2(p[c].x - M);
+        lse2[i] = M + log2f(Z);
+    }
 }
 
 // ---------------------------------------------------------------------------
 // Phase 2 (rows resident): raw_j = sum_r 2^{x_rj - lse_r} for keys of one chunk
 // of [0, P).  Block = (unit, chunk) flattened as u * nchunks + chunk.
 template <int D, int MAX_NTW>
-__global__ void __launch_bounds__(kThreads)
-colsum_rows_kernel(TensorDesc K, TensorDesc Q, Geometry g, int chunk_keys, int nchunks,
-                   const float *__restrict__ lse2, float *__restrict__ raw,
-                   const uint32_t *__restrict__ only)
+__device__ void colsum_rows_block(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                                  int chunk_keys, int nchunks, const float *__restrict__ lse2,
+                                  float *__restrict__ raw, int64_t bid)
 {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ float sCol[kThreads / 32][kTileKeys];
-    const int64_t u = blockIdx.x / nchunks;
-    if (only && only[u] != kUnitRecompute)
-        return;
-    const int chunk = (int)(blockIdx.x % nchunks);
+    const int64_t u = bid / nchunks;
+    const int chunk = (int)(bid % nchunks);
     int l, bb, h;
     unit_coords(g, u, l, bb, h);
     const int rows = g.R;
@@ -341,24 +378,36 @@ colsum_rows_kernel(TensorDesc K, TensorDesc Q, Geometry g, int chunk_keys, int n
     }
 }
 
+template <int D, int MAX_NTW>
+__global__ void __launch_bounds__(kThreads)
+colsum_rows_kernel(TensorDesc K, TensorDesc Q, Geometry g, int chunk_keys, int nchunks,
+                   const float *__restrict__ lse2, float *__restrict__ raw, UnitSel us)
+{
+    const int64_t total = vblocks(us, g.U, nchunks);
+    for (int64_t vb = blockIdx.x; vb < total; vb += gridDim.x) {
+        const int64_t bid = vblock_id(us, nchunks, vb);
+        if (vblock_skip(us, bid / nchunks))
+            continue;
+        colsum_rows_block<D, MAX_NTW>(K, Q, g, chunk_keys, nchunks, lse2, raw, bid);
+        __syncthreads();
+    }
+}
+
 // ---------------------------------------------------------------------------
 // Phase 2 (keys resident, rows streamed) for H2O: CTA owns kKeyBlock keys,
 // warp w owns keys [16w, 16w + 16) with its A fragments in registers, and the
 // rows that can see those keys (position >= first key) stream through smem.
 // Block = (unit, key block) flattened as u * nkb + kb.
 template <int D>
-__global__ void __launch_bounds__(kThreads)
-colsum_keys_kernel(TensorDesc K, TensorDesc Q, Geometry g, int nkb,
-                   const float *__restrict__ lse2, float *__restrict__ raw,
-                   const uint32_t *__restrict__ only)
+__device__ void colsum_keys_block(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                                  int nkb, const float *__restrict__ lse2,
+                                  float *__restrict__ raw, int64_t bid)
 {
     extern __shared__ __align__(16) uint8_t smem[];
     __shared__ float sL[2][kRowTile];
     __shared__ int sPos[2][kRowTile];
-    const int64_t u = blockIdx.x / nkb;
-    const int kb = (int)(blockIdx.x % nkb);
-    if (only && only[u] != kUnitRecompute)
-        return;
+    const int64_t u = bid / nkb;
+    const int kb = (int)(bid % nkb);
     int l, bb, h;
     unit_coords(g, u, l, bb, h);
     const int k_lo = kb * kKeyBlock;
@@ -439,6 +488,38 @@ colsum_keys_kernel(TensorDesc K, TensorDesc Q, Geometry g, int nkb,
     }
 }
 
+template <int D>
+__global__ void __launch_bounds__(kThreads)
+colsum_keys_kernel(TensorDesc K, TensorDesc Q, Geometry g, int nkb,
+                   const float *__restrict__ lse2, float *__restrict__ raw, UnitSel us)
+{
+    const int64_t total = vblocks(us, g.U, nkb);
+    for (int64_t vb = blockIdx.x; vb < total; vb += gridDim.x) {
+        const int64_t bid = vblock_id(us, nkb, vb);
+        if (vblock_skip(us, bid / nkb))
+            continue;
+        colsum_keys_block<D>(K, Q, g, nkb, lse2, raw, bid);
+        __syncthreads();
+    }
+}
+
+// The units flagged kUnitRecompute, as a list (units[0] = count, then the ids in any order:
+// every unit is recomputed on its own).  One CTA.
+__global__ void collect_units_kernel(const uint32_t *__restrict__ flags, int64_t U,
+                                     uint32_t *__restrict__ units)
+{
+    __shared__ uint32_t count;
+    if (threadIdx.x == 0)
+        count = 0;
+    __syncthreads();
+    for (int64_t u = threadIdx.x; u < U; u += blockDim.x)
+        if (flags[u] == kUnitRecompute)
+            units[1 + atomicAdd(&count, 1u)] = (uint32_t)u;
+    __syncthreads();
+    if (threadIdx.x == 0)
+        units[0] = count;
+}
+
 // ---------------------------------------------------------------------------
 // Host launchers.
 
@@ -472,12 +553,12 @@ static cudaError_t prepare(KernelT kernel, size_t smem)
 
 cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int rows_per_block, int chunk_keys, float2 *partial,
-                               cudaStream_t stream, const uint32_t *only)
+                               cudaStream_t stream, UnitSel units)
 {
     const int nrb = (g.R + rows_per_block - 1) / rows_per_block;
     const int nchunks = (g.n + chunk_keys - 1) / chunk_keys;
     const int rows_pad = (min(rows_per_block, g.R) + 7) & ~7;
-    const int64_t blocks = g.U * nrb * nchunks;
+    const int64_t blocks = grid_for(units, g.U * nrb * nchunks);
     cudaError_t err = cudaSuccess;
     const int bucket = max_ntw_bucket(rows_pad);
     if (g.d == 128) {
@@ -487,7 +568,7 @@ cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const G
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
                                  K, Q, g, rows_per_block, nrb, chunk_keys, nchunks, partial,
-                                 only);
+                                 units);
                              err = cudaGetLastError();
                          })
     } else {
@@ -497,7 +578,7 @@ cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const G
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
                                  K, Q, g, rows_per_block, nrb, chunk_keys, nchunks, partial,
-                                 only);
+                                 units);
                              err = cudaGetLastError();
                          })
     }
@@ -505,23 +586,23 @@ cudaError_t launch_lse_partial(const TensorDesc &K, const TensorDesc &Q, const G
 }
 
 cudaError_t launch_combine_lse(const float2 *partial, int64_t total_rows, int nchunks,
-                               float *lse2, cudaStream_t stream, const uint32_t *only,
+                               float *lse2, cudaStream_t stream, UnitSel units,
                                int rows_per_unit)
 {
     const int threads = 256;
-    const int64_t blocks = (total_rows + threads - 1) / threads;
+    const int64_t blocks = grid_for(units, (total_rows + threads - 1) / threads);
     combine_lse_kernel<<<(unsigned)blocks, threads, 0, stream>>>(partial, total_rows, nchunks,
-                                                                  lse2, only, rows_per_unit);
+                                                                  lse2, units, rows_per_unit);
     return cudaGetLastError();
 }
 
 cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                int chunk_keys, const float *lse2, float *raw,
-                               cudaStream_t stream, const uint32_t *only)
+                               cudaStream_t stream, UnitSel units)
 {
     const int nchunks = (g.P + chunk_keys - 1) / chunk_keys;
     const int rows_pad = (g.R + 7) & ~7;
-    const int64_t blocks = g.U * nchunks;
+    const int64_t blocks = grid_for(units, g.U * nchunks);
     cudaError_t err = cudaSuccess;
     const int bucket = max_ntw_bucket(rows_pad);
     if (g.d == 128) {
@@ -530,7 +611,7 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
                          err = prepare(k, smem);
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
-                                 K, Q, g, chunk_keys, nchunks, lse2, raw, only);
+                                 K, Q, g, chunk_keys, nchunks, lse2, raw, units);
                              err = cudaGetLastError();
                          })
     } else {
@@ -539,7 +620,7 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
                          err = prepare(k, smem);
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(
-                                 K, Q, g, chunk_keys, nchunks, lse2, raw, only);
+                                 K, Q, g, chunk_keys, nchunks, lse2, raw, units);
                              err = cudaGetLastError();
                          })
     }
@@ -548,10 +629,10 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
 
 cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
                                const float *lse2, float *raw, cudaStream_t stream,
-                               const uint32_t *only)
+                               UnitSel units)
 {
     const int nkb = (g.P + kKeyBlock - 1) / kKeyBlock;
-    const int64_t blocks = g.U * nkb;
+    const int64_t blocks = grid_for(units, g.U * nkb);
     cudaError_t err;
     if (g.d == 128) {
         const size_t smem = (size_t)(kKeyBlock + 2 * kRowTile) * Pad<128>::kStride * 2;
@@ -559,15 +640,22 @@ cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const G
         if (err != cudaSuccess)
             return err;
         colsum_keys_kernel<128><<<(unsigned)blocks, kThreads, smem, stream>>>(K, Q, g, nkb, lse2,
-                                                                              raw, only);
+                                                                              raw, units);
     } else {
         const size_t smem = (size_t)(kKeyBlock + 2 * kRowTile) * Pad<64>::kStride * 2;
         err = prepare(colsum_keys_kernel<64>, smem);
         if (err != cudaSuccess)
             return err;
         colsum_keys_kernel<64><<<(unsigned)blocks, kThreads, smem, stream>>>(K, Q, g, nkb, lse2,
-                                                                             raw, only);
+                                                                             raw, units);
     }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_collect_units(const uint32_t *flags, int64_t U, uint32_t *units,
+                                 cudaStream_t stream)
+{
+    collect_units_kernel<<<1, 1024, 0, stream>>>(flags, U, units);
     return cudaGetLastError();
 }
 
