@@ -473,51 +473,69 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
             };
             if (warp == 2 && a.phase == 2) {
                 // ---- -lse of every streamed query block, per row: -inf past the cache ------
-                int64_t nb = 0;      // blocks staged so far: slot (nb / kLseGroup) % kLseSlots
+                // A group of kLseGroup blocks (they may straddle tasks) at a time: every lse of
+                // the group is copied to shared memory asynchronously, all in flight at once
+                // (one L2 round trip per group), then each lane negates its own entries.
                 int hd[kLseLoads];   // query head of each of this lane's rows
 #pragma unroll
                 for (int j = 0; j < kLseLoads; ++j)
                     hd[j] = (lane + 32 * j) / a.pb;
-                for (int64_t item = blockIdx.x; !dead && item < a.items; item += S) {
-                    Task T;
+                int64_t item = blockIdx.x;   // cursor: block i of task `item`
+                int i = 0;
+                Task T;
+                bool more = item < a.items;
+                if (more)
                     get_task(a, item, T);
-                    const float *src = a.lse2 + T.u * g.R;
-                    for (int i = 0; i < T.ntiles; ++i, ++nb) {
-                        const int sub = (int)(nb % kLseGroup);
-                        const int slot = (int)((nb / kLseGroup) % kLseSlots);
-                        const uint32_t lph = (uint32_t)((nb / (kLseGroup * kLseSlots)) & 1);
-                        if (sub == 0 && !wait_w(&sm.bar[kBarLseEmpty + slot], lph ^ 1))
-                            break;
+                uint32_t copied[kLseGroup];  // per block: bit j = this lane's row lane + 32 j
+                for (int64_t grp = 0; more && !dead; ++grp) {
+                    const int slot = (int)(grp % kLseSlots);
+                    if (!wait_w(&sm.bar[kBarLseEmpty + slot],
+                                (uint32_t)((grp / kLseSlots) & 1) ^ 1))
+                        break;
+                    float *L = sm.lse + slot * kLseGroup * kLseBlock;
+#pragma unroll
+                    for (int c = 0; c < kLseGroup; ++c) {
+                        copied[c] = 0;
+                        if (!more)
+                            continue;
+                        const float *src = a.lse2 + T.u * g.R;
                         const int p0 = (T.first + i) * a.pb;
-                        float *L = sm.lse + (slot * kLseGroup + sub) * kLseBlock;
-                        // All of a lane's loads in flight at once: one L2 round trip a block.
-                        float v[kLseLoads];
 #pragma unroll
                         for (int j = 0; j < kLseLoads; ++j) {
                             const int r = lane + 32 * j;
-                            const int gh = hd[j];
-                            const int pos = p0 + r - gh * a.pb;
-                            v[j] = (r < a.rows && pos < g.n)
-                                       ? -__ldg(src + (int64_t)gh * g.n + pos)
-                                       : -INFINITY;
+                            const int pos = p0 + r - hd[j] * a.pb;
+                            float *dst = L + c * kLseBlock + r;
+                            if (r < a.rows && pos < g.n) {
+                                asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                                                 ptx::smem_addr(dst)),
+                                             "l"(src + (int64_t)hd[j] * g.n + pos)
+                                             : "memory");
+                                copied[c] |= 1u << j;
+                            } else if (r < a.r_pad) {
+                                *dst = -INFINITY;
+                            }
                         }
-#pragma unroll
-                        for (int j = 0; j < kLseLoads; ++j)
-                            if (lane + 32 * j < a.r_pad)
-                                L[lane + 32 * j] = v[j];
-                        if (sub == kLseGroup - 1) {
-                            __syncwarp();
-                            if (lane == 0)
-                                ptx::mbar_arrive(&sm.bar[kBarLseFull + slot]);
+                        if (++i == T.ntiles) {
+                            i = 0;
+                            item += S;
+                            more = item < a.items;
+                            if (more)
+                                get_task(a, item, T);
                         }
                     }
-                }
-                // A last, partly filled group.
-                if (!dead && nb % kLseGroup != 0) {
+                    asm volatile("cp.async.wait_all;" ::: "memory");
+#pragma unroll
+                    for (int c = 0; c < kLseGroup; ++c)
+#pragma unroll
+                        for (int j = 0; j < kLseLoads; ++j)
+                            if (copied[c] >> j & 1u) {
+                                float *dst = L + c * kLseBlock + lane + 32 * j;
+                                *dst = -*dst;
+                            }
+                    // A last group may be partly filled: its consumers stop at the last block.
                     __syncwarp();
                     if (lane == 0)
-                        ptx::mbar_arrive(
-                            &sm.bar[kBarLseFull + (int)((nb / kLseGroup) % kLseSlots)]);
+                        ptx::mbar_arrive(&sm.bar[kBarLseFull + slot]);
                 }
             } else if (warp == 3 && a.phase == 1) {
                 // ---- row sums of a query block -> lse_r ---------------------------------------

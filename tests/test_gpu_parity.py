@@ -68,6 +68,12 @@ SMALL = {
     "sinks_scored": WL["c1_tiny"].with_(sinks=4, budgets=(100,)),
     "no_pool": WL["c1_tiny"].with_(pool=inputs.POOL_NONE, pool_kernel=1),
     "long_p": WL["c1_tiny"].with_(n=33500, budgets=(600,), n_spans=0),  # P > 32768
+    # the fused pooling reads whole 128-position chunks: P = 32768 exactly (the largest fused
+    # row, no partial chunk) and P = 129 (one chunk and one position)
+    "p_32768": WL["c1_tiny"].with_(n=32778, budgets=(700,), n_spans=0),
+    "p_129": WL["c1_tiny"].with_(n=139, budgets=(60,), n_spans=0),
+    "p_32768_avg": WL["c1_tiny"].with_(n=32778, budgets=(700,), n_spans=0,
+                                       pool=inputs.POOL_AVG),
     "avg_pool_31": WL["c1_tiny"].with_(pool=inputs.POOL_AVG, pool_kernel=31),
     "max_pool_3_d128": WL["c1_tiny"].with_(d=128, pool_kernel=3),
     "gqa8_ragged": WL["c1_tiny"].with_(Hq=16, Hkv=2, n=2117, budgets=(333,)),
@@ -118,7 +124,7 @@ def test_runs_are_bit_identical():
 
 
 @pytest.mark.parametrize("name", ["c2_small", "c3_small", "no_pool", "keep_none", "keep_all",
-                                  "long_p"])
+                                  "long_p", "p_32768", "p_32768_avg", "p_129"])
 def test_separate_calls_match_fused(name):
     """dge_score -> dge_select -> dge_compact equals dge_evict, bit for bit.
 
