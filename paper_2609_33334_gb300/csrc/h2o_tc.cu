@@ -692,50 +692,44 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                     const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
                     const int p0 = (T.first + i) * a.pb;
                     const bool diag = p0 < k0 + kTile;  // some row precedes some key
-                    float nL[kMaxGroups][16];
                     const int sub = (int)(nb % kLseGroup);
                     const int slot = (int)((nb / kLseGroup) % kLseSlots);
                     if (sub == 0)
                         lse_ok = wait_uniform(&sm.bar[kBarLseFull + slot],
                                               (uint32_t)((nb / (kLseGroup * kLseSlots)) & 1));
                     ++nb;
-                    if (lse_ok) {
-                        const float4 *L4 = reinterpret_cast<const float4 *>(
-                            sm.lse + (slot * kLseGroup + sub) * kLseBlock + col_base);
-#pragma unroll
-                        for (int gi = 0; gi < kMaxGroups; ++gi)
-#pragma unroll
-                            for (int q = 0; q < 4; ++q) {
-                                const float4 f = gi < ng ? L4[gi * 4 + q]
-                                                         : make_float4(-INFINITY, -INFINITY,
-                                                                       -INFINITY, -INFINITY);
-                                nL[gi][4 * q] = f.x;
-                                nL[gi][4 * q + 1] = f.y;
-                                nL[gi][4 * q + 2] = f.z;
-                                nL[gi][4 * q + 3] = f.w;
-                            }
-                        if (sub == kLseGroup - 1) {
-                            __syncwarp();
-                            if (lane == 0)
-                                ptx::mbar_arrive(&sm.bar[kBarLseEmpty + slot]);
-                        }
-                    } else {
-#pragma unroll
-                        for (int gi = 0; gi < kMaxGroups; ++gi)
-#pragma unroll
-                            for (int c = 0; c < 16; ++c)
-                                nL[gi][c] = -INFINITY;
-                    }
                     if (acquire_acc(ab, aph)) {
                         const uint32_t tbase =
                             tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
-                        for_groups(tbase, ng, [&](int gi, const float(&v)[16]) {
+                        const float4 *L4 = reinterpret_cast<const float4 *>(
+                            sm.lse + (slot * kLseGroup + sub) * kLseBlock + col_base);
+                        // Per 16-column group: the TMEM read and the group's -lse (shared
+                        // memory) in flight together.
 #pragma unroll
-                            for (int gj = 0; gj < kMaxGroups; ++gj)
-                                if (gj == gi)
-                                    col_add(acc, v, nL[gj], s2, diag, key, p0, a.pb,
-                                            col_base + gj * 16);
-                        });
+                        for (int gi = 0; gi < kMaxGroups; ++gi)
+                            if (gi < ng) {
+                                float v[16], nl[16];
+                                ptx::tmem_ld16(tbase + gi * 16, v);
+#pragma unroll
+                                for (int q = 0; q < 4; ++q) {
+                                    const float4 f = lse_ok ? L4[gi * 4 + q]
+                                                            : make_float4(-INFINITY, -INFINITY,
+                                                                          -INFINITY, -INFINITY);
+                                    nl[4 * q] = f.x;
+                                    nl[4 * q + 1] = f.y;
+                                    nl[4 * q + 2] = f.z;
+                                    nl[4 * q + 3] = f.w;
+                                }
+                                ptx::tmem_ld_wait_dep(v);
+                                col_add(acc, v, nl, s2, diag, key, p0, a.pb, col_base + gi * 16);
+                            }
+                    }
+                    // Every warp has read this block's -lse: the fourth block of a group frees
+                    // the slot.
+                    if (lse_ok && sub == kLseGroup - 1) {
+                        __syncwarp();
+                        if (lane == 0)
+                            ptx::mbar_arrive(&sm.bar[kBarLseEmpty + slot]);
                     }
                     release_acc(ab);
                 }
