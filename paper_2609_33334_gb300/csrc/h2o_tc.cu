@@ -6,8 +6,8 @@
 // In base 2:
 //   x_rj = log2(e) * scale * q_r . k_j,   row r = (g, p) sees keys j <= p,
 //   lse_r = log2 sum_{j <= p} 2^{x_rj},   raw_j = sum_{r : p_r >= j} 2^{x_rj - lse_r}.
-// A unit's rows form query blocks of pb positions x G heads (stacked head-major, at most 144
-// rows: one 5-D TMA box).  Two launches of one persistent, warp-specialised kernel, one CTA
+// A unit's rows form query blocks of pb positions x G heads (stacked head-major, one 5-D TMA
+// box; at most 128 rows in phase 1 and 144 in phase 2).  Two launches of one persistent, warp-specialised kernel, one CTA
 // per SM, tasks dealt round-robin:
 //   phase 1, task (unit, query block): the block stays in shared memory while the key tiles it
 //     can see stream through a ring; the epilogue keeps every row's sum of 2^x in registers,
@@ -17,7 +17,8 @@
 //     keeps one key's column sum for the whole task, and the three warpgroups' partial sums
 //     meet once, at the end of the task.
 // Both phases compute D[128 keys x R_pad rows] = K_tile . Q_block^T with tcgen05.mma (M = 128,
-// bf16 -> fp32) into one of three TMEM accumulators: warp 0 issues the TMA copies, warp 1 the
+// bf16 -> fp32) into one of four (phase 1) or three (phase 2) TMEM accumulators: warp 0 issues
+// the TMA copies, warp 1 the
 // MMAs, warps 4..15 (three warpgroups, a third of the columns each, one key per thread) read
 // the accumulators.  Row sums carry no running maximum: fp32 holds 2^x for |x| < 126, and a
 // unit whose sums leave [2^-60, 2^126) is flagged (ready = 2) and recomputed by the
@@ -48,8 +49,17 @@ static_assert(4 * 32 * kRegsControl + kEpiWarps * 32 * kRegsEpilogue <= kThreads
               "register split");
 constexpr int kMaxGroups = 3;             // 16-column groups per epilogue warpgroup
 constexpr int kMaxBlockRows = kEpiWG * kMaxGroups * 16;
+// Rows of a query block and TMEM accumulators, per phase: phase 1 takes blocks of up to 128
+// rows (four accumulators of 128 columns, so its MMAs run one more tile ahead of the
+// epilogue), phase 2 blocks of up to 144 rows (three of 160 columns).  Measured at c4 with
+// 128-row blocks: phase 1 101 -> 85 ms, phase 2 96.5 -> 103.6 ms (12 % more tiles for it).
+constexpr int kBlockRows1 = 128, kAccBufs1 = 4;
+constexpr int kBlockRows2 = kMaxBlockRows, kAccBufs2 = 3;
+constexpr int kMaxAccBufs = 4;
+static_assert(kAccBufs1 * ((kBlockRows1 + 31) & ~31) <= 512 &&
+                  kAccBufs2 * ((kBlockRows2 + 31) & ~31) <= 512,
+              "TMEM columns");
 constexpr int kStages = 4;                // streamed operand ring
-constexpr int kAccBufs = 3;               // TMEM accumulators
 constexpr int kTmemCols = 512;
 constexpr int kKSlab = kTile * 128;       // 128 keys x 64 bf16
 constexpr int kXchBufs = 4;               // phase-2 end-of-task exchange areas
@@ -58,13 +68,15 @@ constexpr int kXchBufs = 4;               // phase-2 end-of-task exchange areas
 constexpr int kLseGroup = 4;
 constexpr int kLseSlots = 2;
 constexpr int kLseBlock = 160;            // floats per block (>= rows, 16-byte multiple)
-constexpr int kLseLoads = (kMaxBlockRows + 31) / 32;   // staged rows per lane
+constexpr int kLseLoads = (kBlockRows2 + 31) / 32;     // staged rows per lane (phase 2)
 constexpr uint32_t kReadyBad = 2;
 
 // Barrier slots.
 constexpr int kBarRingFull = 0, kBarRingEmpty = 4, kBarStatFull = 8, kBarStatEmpty = 10,
-              kBarAccFull = 12, kBarAccEmpty = 15, kBarDrain = 18, kBarRedFull = 19,
-              kBarRedEmpty = 21, kBarLseFull = 23, kBarLseEmpty = 27, kBarXch = 31,
+              kBarAccFull = 12, kBarAccEmpty = kBarAccFull + kMaxAccBufs,
+              kBarDrain = kBarAccEmpty + kMaxAccBufs, kBarRedFull = kBarDrain + 1,
+              kBarRedEmpty = kBarRedFull + 2, kBarLseFull = kBarRedEmpty + 2,
+              kBarLseEmpty = kBarLseFull + kLseSlots, kBarXch = kBarLseEmpty + kLseSlots,
               kNumBars = kBarXch + kXchBufs * 4;
 constexpr int kCtrlBytes = 512;           // barriers, TMEM address, flags (16-byte multiple)
 // Flag slots (ints): abort, then the parity of the last arm of every ring stage and
@@ -248,7 +260,7 @@ __device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
         }
 }
 
-template <bool kPaged>
+template <bool kPaged, int kAccBufs>
 __global__ void __launch_bounds__(kThreads, 1)
 h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmQ,
               const __grid_constant__ CUtensorMap tmKm, const H2oArgs a)
@@ -789,7 +801,7 @@ bool h2o_tc_supported(const Geometry &g)
         return false;
     // At least 16 positions per block: the causal mask of a 16-column group then wraps to the
     // next head at most once, and every block keeps the tensor pipe busy.
-    if (kMaxBlockRows / g.G < 16)
+    if (kBlockRows1 / g.G < 16 || kBlockRows2 / g.G < 16)
         return false;
     int dev = 0, major = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -801,19 +813,20 @@ bool h2o_tc_supported(const Geometry &g)
 H2oPlan h2o_tc_plan(const Geometry &g)
 {
     H2oPlan p;
-    p.pb = kMaxBlockRows / g.G;
-    if (p.pb > g.n)
-        p.pb = g.n;
-    p.rows = g.G * p.pb;
-    p.r_pad = (p.rows + 15) & ~15;
     p.nslab = g.d / 64;
-    p.nqb = (g.n + p.pb - 1) / p.pb;
     p.nkt = (g.P + kTile - 1) / kTile;
     for (int ph = 1; ph <= 2; ++ph) {
-        size_t s = smem_bytes(ph, p.r_pad, p.nslab);
+        H2oPhase &q = p.ph[ph - 1];
+        q.pb = (ph == 1 ? kBlockRows1 : kBlockRows2) / g.G;
+        if (q.pb > g.n)
+            q.pb = g.n;
+        q.rows = g.G * q.pb;
+        q.r_pad = (q.rows + 15) & ~15;
+        q.nqb = (g.n + q.pb - 1) / q.pb;
+        const size_t s = smem_bytes(ph, q.r_pad, p.nslab);
         // At least half of the SM's shared memory: one CTA per SM, so a CTA's TMEM
         // allocation (all 512 columns) never waits for another CTA of this kernel.
-        p.smem[ph - 1] = s < 120 * 1024 ? 120 * 1024 : s;
+        q.smem = s < 120 * 1024 ? 120 * 1024 : s;
     }
     return p;
 }
@@ -826,7 +839,7 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
     memset(&tmKm, 0, sizeof tmKm);
     const bool merged = K.bt && tc::encode_k_merged_map(&tmKm, K, g.L, g.Hkv, g.d);
     *encoded = tc::encode_k_map(&tmK, K, g.L, g.b, g.Hkv, g.n, g.d) &&
-               tc::encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.n, g.d, plan.pb, g.G);
+               tc::encode_5d(&tmQ, Q, g.L, g.b, g.Hq, g.n, g.d, plan.ph[phase - 1].pb, g.G);
     if (!*encoded)
         return cudaSuccess;
     int dev = 0, sms = 0;
@@ -840,16 +853,17 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
     a.g = g;
     a.kp = tc::k_paging(K, g.n);
     a.kp.merged = merged ? 1 : 0;
+    const H2oPhase &q = plan.ph[phase - 1];
     a.phase = phase;
-    a.pb = plan.pb;
-    a.rows = plan.rows;
-    a.r_pad = plan.r_pad;
+    a.pb = q.pb;
+    a.rows = q.rows;
+    a.r_pad = q.r_pad;
     a.nslab = plan.nslab;
-    a.acc_stride = (plan.r_pad + 31) & ~31;
-    a.nqb = plan.nqb;
+    a.acc_stride = (q.r_pad + 31) & ~31;
+    a.nqb = q.nqb;
     a.nkt = plan.nkt;
-    a.items = g.U * (phase == 1 ? (int64_t)plan.nqb : (int64_t)plan.nkt);
-    const int NG = plan.r_pad / 16;
+    a.items = g.U * (phase == 1 ? (int64_t)q.nqb : (int64_t)plan.nkt);
+    const int NG = q.r_pad / 16;
     for (int w = 0, base = 0; w < kEpiWG; ++w) {
         a.ng[w] = NG / kEpiWG + (w < NG % kEpiWG ? 1 : 0);
         a.gbase[w] = base;
@@ -862,8 +876,9 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
     a.timeout_ns = 4000000000ull;
     if (a.items == 0)
         return cudaSuccess;
-    const size_t smem = plan.smem[phase - 1];
-    auto kernel = K.bt ? h2o_tc_kernel<true> : h2o_tc_kernel<false>;
+    const size_t smem = q.smem;
+    auto kernel = phase == 1 ? (K.bt ? h2o_tc_kernel<true, kAccBufs1> : h2o_tc_kernel<false, kAccBufs1>)
+                             : (K.bt ? h2o_tc_kernel<true, kAccBufs2> : h2o_tc_kernel<false, kAccBufs2>);
     err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (err != cudaSuccess)
         return err;

@@ -61,14 +61,17 @@ cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const G
                                UnitSel units = {});
 
 // H2O scoring on the tcgen05 path (h2o_tc.cu): query blocks of pb positions x G heads.
-struct H2oPlan {
+struct H2oPhase {
     int pb;            // positions per query block
     int rows;          // G * pb stacked rows of a block
     int r_pad;         // rows rounded up to 16 (the MMA's N)
-    int nslab;         // d / 64
     int nqb;           // query blocks per unit
+    size_t smem;       // dynamic shared memory
+};
+struct H2oPlan {
+    H2oPhase ph[2];    // phase 1 (row normalisers), phase 2 (column sums)
+    int nslab;         // d / 64
     int nkt;           // 128-key tiles of past keys per unit
-    size_t smem[2];    // dynamic shared memory of phase 1 / phase 2
 };
 bool h2o_tc_supported(const Geometry &g);
 H2oPlan h2o_tc_plan(const Geometry &g);

@@ -78,8 +78,9 @@ SMALL = {
     "max_pool_3_d128": WL["c1_tiny"].with_(d=128, pool_kernel=3),
     "gqa8_ragged": WL["c1_tiny"].with_(Hq=16, Hkv=2, n=2117, budgets=(333,)),
     "h2o_tiny": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=4, Hkv=2, d=64, n=300, budgets=(100,)),
-    # H2O query blocks: G = 5 gives 28 positions x 5 heads = 140 rows (4 padded columns),
-    # G = 8 gives 18 positions, G = 1 a single 144-position block of one head
+    # H2O query blocks (phase 1 / phase 2): G = 5 gives 25 / 28 positions x 5 heads = 125 / 140
+    # rows (3 / 4 padded columns), G = 8 gives 16 / 18 positions, G = 1 single-head blocks of
+    # 128 / 144 positions
     "h2o_g5_padded": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=10, Hkv=2, d=64, n=777, budgets=(200,)),
     "h2o_g8": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=16, Hkv=2, n=500, budgets=(150,)),
     "h2o_g1": WL["c4_h2o_8k"].with_(L=2, b=1, Hq=2, Hkv=2, n=403, budgets=(120, 90)),
