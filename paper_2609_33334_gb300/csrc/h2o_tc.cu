@@ -224,9 +224,12 @@ __device__ __forceinline__ void rows_add(float (&z)[16], const float (&v)[16], f
 }
 
 // Phase 2 for one 16-column group: adds 2^{x_c - lse_c} over the rows that see `key`.  nL
-// holds -lse (rows past the cache or padding: -inf).
-__device__ __forceinline__ void col_add(float2 &acc, const float (&v)[16], const float (&nL)[16],
-                                        float s2, bool diag, int key, int p0, int pb, int cb)
+// holds -lse (rows past the cache or padding: -inf).  Columns 2q, 2q+1 go to acc[q % 4]: four
+// independent chains of additions instead of one (the epilogue is latency-bound), added
+// together in a fixed order at the end of the task.
+__device__ __forceinline__ void col_add(float2 (&acc)[4], const float (&v)[16],
+                                        const float (&nL)[16], float s2, bool diag, int key,
+                                        int p0, int pb, int cb)
 {
     if (!diag) {
         const float2 sc = make_float2(s2, s2);
@@ -234,14 +237,14 @@ __device__ __forceinline__ void col_add(float2 &acc, const float (&v)[16], const
         for (int c = 0; c < 16; c += 2) {
             const float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc,
                                         make_float2(nL[c], nL[c + 1]));
-            acc = __fadd2_rn(acc, make_float2(ex2(x.x), ex2(x.y)));
+            acc[(c >> 1) & 3] = __fadd2_rn(acc[(c >> 1) & 3], make_float2(ex2(x.x), ex2(x.y)));
         }
     } else {
         const uint32_t mask = causal_mask(key, p0, pb, cb);
 #pragma unroll
         for (int c = 0; c < 16; ++c) {
             const float p = ex2(v[c] * s2 + nL[c]);
-            acc.x += ((mask >> c) & 1u) ? p : 0.f;
+            acc[(c >> 1) & 3].x += ((mask >> c) & 1u) ? p : 0.f;
         }
     }
 }
@@ -698,7 +701,10 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                 get_task(a, item, T);
                 const int k0 = T.blk * kTile;
                 const int key = k0 + kl;
-                float2 acc = make_float2(0.f, 0.f);
+                float2 acc[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    acc[q] = make_float2(0.f, 0.f);
                 for (int i = 0; i < T.ntiles; ++i, ++tc) {
                     const int ab = tc % kAccBufs;
                     const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
@@ -753,7 +759,9 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                 const int xb = xc % kXchBufs;
                 ++xc;
                 float *xs = sm.xch + xb * kEpiWG * kTile;
-                xs[wg * kTile + kl] = acc.x + acc.y;
+                xs[wg * kTile + kl] =
+                    ((acc[0].x + acc[0].y) + (acc[1].x + acc[1].y)) +
+                    ((acc[2].x + acc[2].y) + (acc[3].x + acc[3].y));
                 __syncwarp();
                 int last = 0;
                 if (lane == 0) {
