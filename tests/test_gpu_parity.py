@@ -84,6 +84,8 @@ SMALL = {
     "h2o_g5_padded": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=10, Hkv=2, d=64, n=777, budgets=(200,)),
     "h2o_g8": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=16, Hkv=2, n=500, budgets=(150,)),
     "h2o_g1": WL["c4_h2o_8k"].with_(L=2, b=1, Hq=2, Hkv=2, n=403, budgets=(120, 90)),
+    # G = 9: fewer than 16 positions per 128-row block, so the warp-level kernels score it
+    "h2o_g9": WL["c4_h2o_8k"].with_(L=1, b=1, Hq=18, Hkv=2, d=64, n=300, budgets=(100,)),
     "slm_keep_all": WL["c5_slm"].with_(L=1, n=300, Hq=8, Hkv=2, budgets=(300,), n_spans=0),
 }
 
@@ -247,6 +249,16 @@ def test_tensor_core_path_is_taken_where_eligible(name, kernel):
     names = _kernels_run(lambda: api.evict(p, tens["K"], tens["V"], tens["Q"]))
     assert kernel in names, names
     assert "colsum_rows" not in names and "colsum_keys" not in names, names
+
+
+def test_h2o_large_groups_take_the_warp_level_kernels():
+    """H2O with G = 9 cannot form 16-position query blocks: it is scored by the warp-level
+    kernels (and matches the oracle in test_small_cases_match_oracle)."""
+    wl = SMALL["h2o_g9"]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    names = _kernels_run(lambda: api.evict(p, tens["K"], tens["V"], tens["Q"]))
+    assert "colsum_keys" in names and not any(n.startswith("h2o_tc") for n in names), names
 
 
 def test_paths_agree_closely():
