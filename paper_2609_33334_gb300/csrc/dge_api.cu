@@ -512,13 +512,15 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
         if (rc != DGE_OK || done)
             return rc;
     }
-    DGE_LAUNCH("lse_partial", stream, launch_lse_partial(K, Q, g, plan.rows_per_block, plan.chunk_keys, partial,
-                                      stream));
-    DGE_LAUNCH("combine_lse", stream, launch_combine_lse(partial, g.U * g.R, plan.nchunks, lse2, stream));
+    DGE_LAUNCH("lse_partial", stream,
+               launch_lse_partial(K, Q, g, plan.rows_per_block, plan.chunk_keys, partial, stream));
+    DGE_LAUNCH("combine_lse", stream,
+               launch_combine_lse(partial, g.U * g.R, plan.nchunks, lse2, stream));
     if (g.variant == DGE_VARIANT_H2O)
         DGE_LAUNCH("colsum_keys", stream, launch_colsum_keys(K, Q, g, lse2, raw, stream));
     else
-        DGE_LAUNCH("colsum_rows", stream, launch_colsum_rows(K, Q, g, kScoredChunkKeys, lse2, raw, stream));
+        DGE_LAUNCH("colsum_rows", stream,
+                   launch_colsum_rows(K, Q, g, kScoredChunkKeys, lse2, raw, stream));
     if (lse_out)
         DGE_LAUNCH("lse_export", stream,
                    launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
@@ -585,8 +587,9 @@ int dge_score(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
     if ((rc = run_scoring(plan, kv_desc(bufs->K, bufs->paging), desc(bufs->Q), ws, stream,
                           bufs->lse_in, bufs->lse_out)) != DGE_OK)
         return rc;
-    DGE_LAUNCH("pool", stream, launch_pool(ws_at<float>(ws, plan.off_raw), bufs->scores, plan.g.U, plan.g.P,
-                               plan.g.pool, plan.g.pool_kernel, stream));
+    DGE_LAUNCH("pool", stream,
+               launch_pool(ws_at<float>(ws, plan.off_raw), bufs->scores, plan.g.U, plan.g.P,
+                           plan.g.pool, plan.g.pool_kernel, stream));
     return DGE_OK;
 }
 
@@ -697,7 +700,8 @@ int evict_impl(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t w
                    launch_pool_select(g, plan.layers, raw, bufs->scores, bufs->idx, stream));
     } else if (g.pool != DGE_POOL_NONE) {
         float *pooled = bufs->scores ? bufs->scores : ws_at<float>(ws, plan.off_pooled);
-        DGE_LAUNCH("pool", stream, launch_pool(raw, pooled, g.U, g.P, g.pool, g.pool_kernel, stream));
+        DGE_LAUNCH("pool", stream,
+                   launch_pool(raw, pooled, g.U, g.P, g.pool, g.pool_kernel, stream));
         sel = pooled;
     } else if (bufs->scores) {
         DGE_CHECK_CUDA(cudaMemcpyAsync(bufs->scores, raw, (size_t)g.U * g.P * sizeof(float),
