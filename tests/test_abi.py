@@ -86,6 +86,20 @@ def test_packed_rows_and_workspace(lib, name):
         assert ws >= p.U * p.P * 4
 
 
+@pytest.mark.parametrize("n", [80, 127, 128, 129, 1000, 3000, 5000, 8192, 32768, 131072])
+@pytest.mark.parametrize("G,m", [(4, 34), (8, 66)])   # whole units (R = 136); 4 row blocks
+def test_workspace_for_cache_lengths_and_row_blocks(lib, n, G, m):
+    """The scoring plan (key chunks of the tensor-core kernel, row blocks) is computed on the
+    host for every problem: every cache length from below one key tile up to 128K keys gives a
+    valid workspace size, with room for the raw scores and the fixed-point row-block sums."""
+    p = _problem(Hq=8 * G, Hkv=8, d=128, n=n, m=m, tail=m, budgets=[min(n, 2 * m)])
+    ws = ctypes.c_size_t(0)
+    assert lib.dge_workspace_size(ctypes.byref(p), ctypes.byref(ws)) == 0
+    U, P = 8, n - m
+    need = U * P * 4 * (3 if G == 8 else 1)   # raw scores (+ 8-byte fixed-point sums)
+    assert ws.value >= need and ws.value % 256 == 0
+
+
 def _problem(**kw):
     base = dict(L=1, b=1, Hq=8, Hkv=2, d=64, n=1024, m=10, tail=10, sinks=0,
                 variant=B.DGE_VARIANT_SCORED, pool=B.DGE_POOL_MAX, pool_kernel=7,
