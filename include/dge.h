@@ -25,9 +25,17 @@
  *       row_base(l) = batch * Hkv * (budgets[0] + ... + budgets[l-1]).
  *     Kc, Vc are [rows][d] bf16, contiguous.  idx rows are ascending positions.
  *   - Every device pointer is caller-owned.  The library allocates no device
- *     memory, keeps no device state between calls, and never synchronises the
- *     caller's stream (except dge_get_device_status).  All work is enqueued on
+ *     memory and never synchronises the caller's stream (except
+ *     dge_get_device_status and dge_noalloc_status).  It keeps no device state
+ *     between calls, with one exception: the fixed scratch array of
+ *     dge_score_noalloc, which is part of the library's device image (every GPU
+ *     that loads the library holds it until exit).  All work is enqueued on
  *     `stream` (a cudaStream_t passed as void*; NULL = legacy default stream).
+ *   - Which scoring kernels run is decided per call from the problem and the
+ *     device (tcgen05 kernels where they apply, warp-level kernels otherwise);
+ *     the environment variable DGE_SCORE_KERNEL=mma, read on every scoring
+ *     call, forces the warp-level kernels (a check of one path against the
+ *     other; the results agree within the score tolerance, not bit for bit).
  *   - Outputs must not alias inputs.
  *   - Validation errors are returned before anything is enqueued.  Launch
  *     failures return DGE_ERR_CUDA; dge_last_error() then holds the CUDA error
@@ -204,17 +212,34 @@ int dge_score(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t ws
  * is rejected with DGE_ERR_WORKSPACE_TOO_SMALL before anything is enqueued
  * (dge_last_error() then states both sizes).  The first call on each device
  * looks up the array's device address with that device current, so make that
- * first call before any stream capture.  Every call uses the same array and it
+ * first call before any stream capture.  The address is kept for the life of
+ * the process: do not use this call on a device after cudaDeviceReset() (the
+ * array may then live elsewhere).  Every call uses the same array and it
  * keeps the previous call's contents (the call itself clears what must start
  * at zero), so calls that can overlap on the GPU -- on different streams or
  * from different host threads -- race; serialise them.  Inputs, outputs and
- * results are those of dge_score.
+ * scores are those of dge_score.  Device-side reports (a bounded wait that
+ * gave up) land in the status word at the start of the built-in array, which
+ * the caller cannot address: read them with dge_noalloc_status before the
+ * next dge_score_noalloc call, which clears the word when it starts.
  */
 #define DGE_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 int dge_score_noalloc(const dge_problem *p, const dge_buffers *bufs, void *stream);
 
 /*
+ * The device status word of dge_score_noalloc's built-in array on the current
+ * device: synchronises `stream`, reads the word, clears it and returns it, as
+ * dge_get_device_status does for a caller's workspace (DGE_OK when nothing
+ * was reported).  Returns DGE_ERR_INVALID_ARG if dge_score_noalloc has not run
+ * on this device.  Allocates nothing.
+ */
+int dge_noalloc_status(void *stream);
+
+/*
  * Retention (Alg. 1: I <- R_E(s, B - w); App. E: sort to keep temporal order).
+ * Takes no workspace: the selection runs in shared memory and reads the scores
+ * from global memory, so it needs no device scratch and reports no
+ * device-side status.
  * For every unit keeps [0, sinks), the budgets[l] - sinks - tail positions of
  * [sinks, P) with the largest scores (equal scores: lower position first), and
  * [P, n); writes them ascending to the packed idx.  STREAMING ignores scores
@@ -372,6 +397,18 @@ int dge_profile_end(dge_kernel_time *out, int capacity, int *count);
 #define DGE_TRACE_SLOTS 24
 #define DGE_TRACE_LEN 4096
 int dge_trace_set(void *buffer, size_t bytes, int cta);
+
+/*
+ * Test hook of the device-side failure detection, off by default.  limit_ns
+ * bounds every later device-side wait of the tcgen05 kernels (0 restores the
+ * default, 4 s).  extra_chunks > 0 makes the tensor-core scoring kernel's wait
+ * for a unit's row sums expect that many key chunks more than exist, so the
+ * wait can only run out: the kernel then records DGE_ERR_DEVICE_TIMEOUT in the
+ * status word, stops, drains its copies and MMAs, frees its tensor memory and
+ * returns (results of that call are undefined; the context stays usable).
+ * Host-side state, per process; not for production use.
+ */
+int dge_debug_set_waits(uint64_t limit_ns, int32_t extra_chunks);
 
 /* Static text for a status code. */
 const char *dge_status_string(int code);

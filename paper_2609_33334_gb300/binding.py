@@ -80,6 +80,7 @@ _SIGS = {
     "dge_packed_rows": [_P, POINTER(c_int64)],
     "dge_score": [_P, _B, c_void_p, c_size_t, c_void_p],
     "dge_score_noalloc": [_P, _B, c_void_p],
+    "dge_noalloc_status": [c_void_p],
     "dge_select": [_P, c_void_p, c_void_p, c_void_p],
     "dge_compact": [_P, c_void_p, _T, _T, c_void_p, c_void_p, c_void_p, c_void_p],
     "dge_evict": [_P, _B, c_void_p, c_size_t, c_void_p],
@@ -94,6 +95,7 @@ _SIGS = {
     "dge_last_error": [],
     "dge_profile_begin": [],
     "dge_trace_set": [c_void_p, c_size_t, c_int],
+    "dge_debug_set_waits": [ctypes.c_uint64, c_int32],
     "dge_profile_end": [POINTER(dge_kernel_time), c_int, POINTER(c_int)],
 }
 
@@ -148,6 +150,11 @@ def dge_score_noalloc(p: dge_problem, bufs: dge_buffers, stream: int) -> None:
     """dge_score with the library's built-in scratch (no workspace, nothing allocated)."""
     _check("dge_score_noalloc", _lib().dge_score_noalloc(ctypes.byref(p), ctypes.byref(bufs),
                                                          stream))
+
+
+def dge_noalloc_status(stream: int) -> int:
+    """Reads and clears the status word of dge_score_noalloc's built-in scratch."""
+    return _lib().dge_noalloc_status(stream)
 
 
 def dge_select(p: dge_problem, scores: int, idx: int, stream: int) -> None:
@@ -230,6 +237,12 @@ def dge_profile_end(capacity: int = 32) -> list:
 
 
 TRACE_SLOTS, TRACE_LEN = 24, 4096
+
+
+def dge_debug_set_waits(limit_ns: int = 0, extra_chunks: int = 0) -> None:
+    """Test hook: bound of the tcgen05 kernels' device-side waits (0 = default) and extra
+    chunks the scoring kernel's unit-count wait expects (> 0: that wait runs out)."""
+    _check("dge_debug_set_waits", _lib().dge_debug_set_waits(limit_ns, extra_chunks))
 
 
 def dge_trace_set(buffer: int, nbytes: int, cta: int = 0) -> None:

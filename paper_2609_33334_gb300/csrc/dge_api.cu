@@ -121,7 +121,8 @@ struct Plan {
     int nchunks = 0;
     TcPlan tc = {};          // tensor-core path decomposition (SCORED only)
     size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, off_count = 0,
-           off_ready = 0, off_rawfx = 0, off_unitflag = 0, off_units = 0, ws_bytes = 0;
+           off_ready = 0, off_rawfx = 0, off_units = 0, off_rpart = 0, ws_bytes = 0;
+    size_t flags_clear = 0;  // bytes from off_count that a tensor-core scoring call zeroes
 };
 
 constexpr int kScoredChunkKeys = 2048;
@@ -248,20 +249,25 @@ int make_plan(const dge_problem *p, Plan &plan)
         plan.off_pooled = off;
         if (g.pool != DGE_POOL_NONE)
             off = align256(off + (size_t)g.U * g.P * sizeof(float));
+        // Flags, one region: chunk counters [U*nrb] (tensor-core path), per-unit range flags
+        // [U], then the list of units to recompute ([0] = count, [1 ..] = ids).  The counters,
+        // the flags and the list count are zeroed with one memset before a scoring launch.
         plan.off_count = off;
-        off = align256(off + (size_t)g.U * nrb * sizeof(uint32_t));
-        plan.off_ready = off;
-        off = align256(off + (size_t)g.U * nrb * sizeof(uint32_t));
-        // Units left for the recompute: count, then ids.
-        plan.off_units = off;
-        off = align256(off + (size_t)(g.U + 1) * sizeof(uint32_t));
+        plan.off_ready = off + (size_t)g.U * nrb * sizeof(uint32_t);
+        plan.off_units = plan.off_ready + (size_t)g.U * sizeof(uint32_t);
+        plan.flags_clear = plan.off_units + sizeof(uint32_t) - plan.off_count;
+        off = align256(plan.off_units + (size_t)(g.U + 1) * sizeof(uint32_t));
         if (nrb > 1) {
             // Row blocks of one unit add their column sums in fixed point (exact, so the
-            // order of the additions does not matter), and their range flags per unit.
+            // order of the additions does not matter).
             plan.off_rawfx = off;
             off = align256(off + (size_t)g.U * g.P * sizeof(unsigned long long));
-            plan.off_unitflag = off;
-            off = align256(off + (size_t)g.U * sizeof(uint32_t));
+        }
+        if (p->variant == DGE_VARIANT_SCORED) {
+            // Row partials of the units recomputed with running maxima ([U][R] float2): apart
+            // from the tensor-core chunk sums, which the normaliser export still reads.
+            plan.off_rpart = off;
+            off = align256(off + (size_t)g.U * g.R * sizeof(float2));
         }
     }
     plan.ws_bytes = off;
@@ -455,54 +461,41 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
         return DGE_OK;
     }
     if (g.variant == DGE_VARIANT_SCORED && want_tc(g)) {
-        uint32_t *count = ws_at<uint32_t>(ws, plan.off_count);
-        uint32_t *ready = ws_at<uint32_t>(ws, plan.off_ready);
-        const size_t nsub = (size_t)g.U * plan.tc.nrb;   // sub-units (row blocks)
-        DGE_CHECK_CUDA(cudaMemsetAsync(count, 0, nsub * sizeof(uint32_t), stream),
-                       "counter clear");
-        DGE_CHECK_CUDA(cudaMemsetAsync(ready, 0, nsub * sizeof(uint32_t), stream), "flag clear");
+        DGE_CHECK_CUDA(cudaMemsetAsync(ws_at<uint8_t>(ws, plan.off_count), 0, plan.flags_clear,
+                                       stream),
+                       "flag clear");
         TcBuffers tb;
         tb.part = reinterpret_cast<float *>(partial);
         tb.lse2 = lse2;
         tb.raw = raw;
-        tb.count = count;
-        tb.ready = ready;
+        tb.count = ws_at<uint32_t>(ws, plan.off_count);
+        tb.ready = ws_at<uint32_t>(ws, plan.off_ready);
+        tb.list = ws_at<uint32_t>(ws, plan.off_units);
         tb.status = static_cast<uint32_t *>(ws);
         const int nrb = plan.tc.nrb;
         unsigned long long *raw_fx = nullptr;
-        uint32_t *unit_flag = ready;      // per-unit range flags for the recompute
         if (nrb > 1) {
             raw_fx = ws_at<unsigned long long>(ws, plan.off_rawfx);
             DGE_CHECK_CUDA(cudaMemsetAsync(raw_fx, 0, (size_t)g.U * g.P * 8, stream),
                            "sum clear");
             tb.raw_fx = raw_fx;
-            unit_flag = ws_at<uint32_t>(ws, plan.off_unitflag);
         }
         bool encoded = false;
         DGE_LAUNCH("score_tc", stream,
                    launch_score_tc(K, Q, g, plan.tc, tb, stream, &encoded));
         if (encoded) {
-            if (nrb > 1) {
+            if (nrb > 1)
                 DGE_LAUNCH("fixed_to_float", stream,
                            launch_fixed_to_float(raw_fx, raw, g.U * g.P, stream));
-                DGE_LAUNCH("unit_flags", stream,
-                           launch_unit_flags(ready, nrb, g.U, unit_flag, stream));
-            }
-            // Units whose row sums left fp32's safe range (flag 2) are recomputed with the
-            // running-maximum kernels; every other unit's CTA returns at once (one CTA per
-            // unit: cheaper than collecting a list first).
-            UnitSel units;
-            units.sel = unit_flag;
-            DGE_LAUNCH("recompute_lse", stream,
-                       launch_lse_partial(K, Q, g, g.R, g.n, partial, stream, units));
-            DGE_LAUNCH("recompute_combine", stream,
-                       launch_combine_lse(partial, g.U * g.R, 1, lse2, stream, units, g.R));
-            DGE_LAUNCH("recompute_colsum", stream,
-                       launch_colsum_rows(K, Q, g, g.P, lse2, raw, stream, units));
+            // Units whose row sums left fp32's safe range were listed by the kernel; one CTA
+            // per listed unit recomputes it with running maxima (an empty list: one read).
+            DGE_LAUNCH("recompute", stream,
+                       launch_recompute_units(K, Q, g, ws_at<float2>(ws, plan.off_rpart), lse2,
+                                              raw, tb.list, stream));
             if (lse_out)
                 DGE_LAUNCH("lse_export", stream,
                            launch_lse_export(tb.part, plan.tc.nchunks, plan.tc.r4, lse2,
-                                             unit_flag, g.U, g.R, plan.tc.rows, lse_out, stream));
+                                             tb.ready, g.U, g.R, plan.tc.rows, lse_out, stream));
             return DGE_OK;
         }
     }
@@ -883,6 +876,14 @@ const char *dge_status_string(int code)
 }
 
 const char *dge_last_error(void) { return g_last_error; }
+
+int dge_debug_set_waits(uint64_t limit_ns, int32_t extra_chunks)
+{
+    if (extra_chunks < 0)
+        return DGE_ERR_INVALID_ARG;
+    tc_set_waits(limit_ns, extra_chunks);
+    return DGE_OK;
+}
 
 int dge_trace_set(void *buffer, size_t bytes, int cta)
 {

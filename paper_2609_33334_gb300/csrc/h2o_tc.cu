@@ -881,7 +881,7 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
     a.raw = raw;
     a.ready = ready;
     a.status = status;
-    a.timeout_ns = 4000000000ull;
+    a.timeout_ns = tc_wait_limit_ns();
     if (a.items == 0)
         return cudaSuccess;
     const size_t smem = q.smem;

@@ -27,6 +27,12 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
 // The units whose flag (flags[U]) equals kUnitRecompute into units[1 + U] (count first).
 cudaError_t launch_collect_units(const uint32_t *flags, int64_t U, uint32_t *units,
                                  cudaStream_t stream);
+// SCORED units of a device-side list (list[0] = count, then ids), each recomputed whole by
+// one CTA with running maxima: row normalisers into lse2 (partial: [U][R] float2 scratch),
+// then the column sums into raw.  A capped grid: an empty list costs one read per CTA.
+cudaError_t launch_recompute_units(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                                   float2 *partial, float *lse2, float *raw, const uint32_t *list,
+                                   cudaStream_t stream);
 
 // Scoring on the tcgen05 path (score_tc.cu).
 struct TcPlan {
@@ -42,14 +48,19 @@ struct TcBuffers {
     float *lse2;       // [U][R]
     float *raw;        // [U][P]
     unsigned long long *raw_fx = nullptr;  // [U][P], nrb > 1: fixed-point sums (2^-40)
-    uint32_t *count;   // [U*nrb], zero before the launch
-    uint32_t *ready;   // [U*nrb], zero before the launch; 2 = recompute
-    uint32_t *status;
+    uint32_t *count = nullptr;  // [U*nrb], zero before the launch
+    uint32_t *ready = nullptr;  // [U], zero before the launch; 2 = recompute
+    uint32_t *list = nullptr;   // [1 + U], list[0] zero before the launch: the units flagged 2
+    uint32_t *status = nullptr;
     const float *lse_in = nullptr;  // [U][R] supplied natural-log normalisers (one pass)
 };
 bool tc_supported(const Geometry &g);
 // Trace buffer of the tensor-core scoring kernel (see dge_trace_set); nullptr = off.
 void tc_set_trace(unsigned long long *buffer, int cta);
+// Test hook (see dge_debug_set_waits): the bound of the tcgen05 kernels' device-side waits
+// (0 = the default) and extra chunks the scoring kernel's unit-count wait expects.
+void tc_set_waits(unsigned long long limit_ns, int count_extra);
+unsigned long long tc_wait_limit_ns();
 TcPlan tc_plan(const Geometry &g);
 // Both phases in one launch.  *encoded is false when the tensors cannot be described
 // to TMA (nothing is launched then).
@@ -91,12 +102,10 @@ cudaError_t launch_lse_import(const float *lse_in, float *lse2, int64_t total, c
 cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const float *lse2,
                               const uint32_t *ready, int64_t U, int R, int rows, float *lse_out,
                               cudaStream_t stream);
-// Fixed-point (2^-40) column sums of row blocks -> float; per-unit range flags from the
-// flags of its nrb row blocks.
+// Fixed-point (2^-40) column sums of row blocks -> float.
 cudaError_t launch_fixed_to_float(const unsigned long long *fx, float *out, int64_t total,
                                   cudaStream_t stream);
-cudaError_t launch_unit_flags(const uint32_t *sub_flag, int nrb, int64_t U, uint32_t *unit_flag,
-                              cudaStream_t stream);
+
 // Diagnostics of one eviction from lse (full cache) and lse_hat (kept keys), both [U][R]
 // natural log: rho_io holds lse_hat on entry and the evicted mass on return; l_match and
 // run_length [U] (nullable).

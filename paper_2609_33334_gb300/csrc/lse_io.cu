@@ -60,19 +60,6 @@ __global__ void fixed_to_float_kernel(const unsigned long long *__restrict__ fx,
         out[i] = __ll2float_rn((long long)fx[i]) * 0x1p-40f;   // one rounding, exact scaling
 }
 
-// A unit is recomputed when any of its row blocks left fp32's range.
-__global__ void unit_flags_kernel(const uint32_t *__restrict__ sub_flag, int nrb, int64_t U,
-                                  uint32_t *__restrict__ unit_flag)
-{
-    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U;
-         u += (int64_t)gridDim.x * blockDim.x) {
-        uint32_t f = 0;
-        for (int rb = 0; rb < nrb; ++rb)
-            f = max(f, sub_flag[u * nrb + rb]);
-        unit_flag[u] = f;
-    }
-}
-
 int blocks_for(int64_t total)
 {
     const int64_t b = (total + 255) / 256;
@@ -103,11 +90,5 @@ cudaError_t launch_fixed_to_float(const unsigned long long *fx, float *out, int6
     return cudaGetLastError();
 }
 
-cudaError_t launch_unit_flags(const uint32_t *sub_flag, int nrb, int64_t U, uint32_t *unit_flag,
-                              cudaStream_t stream)
-{
-    unit_flags_kernel<<<blocks_for(U), 256, 0, stream>>>(sub_flag, nrb, U, unit_flag);
-    return cudaGetLastError();
-}
 
 }  // namespace dge

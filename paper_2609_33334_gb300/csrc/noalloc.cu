@@ -24,8 +24,10 @@ constexpr int kMaxDevices = 64;
 std::mutex g_mu;
 void *g_scratch_addr[kMaxDevices];  // device address of g_noalloc_scratch, per device
 
-// Device address of the scratch on the current device, looked up once per device.
-int scratch_on_current_device(void **out)
+// Device address of the scratch on the current device, looked up once per device (the
+// header asks callers not to use the entry point across a device reset).  With lookup
+// false, only an address already looked up is returned.
+int scratch_on_current_device(void **out, bool lookup = true)
 {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -39,6 +41,8 @@ int scratch_on_current_device(void **out)
         return DGE_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lk(g_mu);
     if (!g_scratch_addr[dev]) {
+        if (!lookup)
+            return DGE_ERR_INVALID_ARG;
         void *ptr = nullptr;
         e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
         if (e != cudaSuccess || !ptr) {
@@ -75,4 +79,15 @@ extern "C" int dge_score_noalloc(const dge_problem *p, const dge_buffers *bufs, 
     if ((rc = scratch_on_current_device(&scratch)) != DGE_OK)
         return rc;
     return dge_score(p, bufs, scratch, kScratchBytes, stream);
+}
+
+// The status word at the start of the scratch (the first 4 bytes of a workspace are the
+// status word for every scoring call), read, cleared and returned like a caller's.
+extern "C" int dge_noalloc_status(void *stream)
+{
+    void *scratch = nullptr;
+    const int rc = scratch_on_current_device(&scratch, false);
+    if (rc != DGE_OK)
+        return rc;
+    return dge_get_device_status(scratch, stream);
 }

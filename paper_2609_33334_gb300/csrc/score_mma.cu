@@ -503,6 +503,31 @@ colsum_keys_kernel(TensorDesc K, TensorDesc Q, Geometry g, int nkb,
     }
 }
 
+// Units of a list (list[0] = count, list[1 ..] = ids), each recomputed whole by one CTA:
+// the row normalisers over all keys with running maxima (one chunk, all rows), then the
+// column sums over [0, P).  The merge of a single chunk is the combine step's: lse = m +
+// log2(z).  The CTA's own global writes of lse2 are visible to it after the barrier.
+template <int D, int MAX_NTW>
+__global__ void __launch_bounds__(kThreads)
+recompute_units_kernel(TensorDesc K, TensorDesc Q, Geometry g, float2 *__restrict__ partial,
+                       float *__restrict__ lse2, float *__restrict__ raw,
+                       const uint32_t *__restrict__ list)
+{
+    const uint32_t count = list[0];
+    for (uint32_t i = blockIdx.x; i < count; i += gridDim.x) {
+        const int64_t u = list[1 + i];
+        lse_partial_block<D, MAX_NTW>(K, Q, g, g.R, 1, g.n, 1, partial, u);
+        __syncthreads();
+        for (int r = threadIdx.x; r < g.R; r += blockDim.x) {
+            const float2 p = partial[u * g.R + r];
+            lse2[u * g.R + r] = p.x + log2f(p.y);
+        }
+        __syncthreads();
+        colsum_rows_block<D, MAX_NTW>(K, Q, g, g.P, 1, lse2, raw, u);
+        __syncthreads();
+    }
+}
+
 // The units flagged kUnitRecompute, as a list (units[0] = count, then the ids in any order:
 // every unit is recomputed on its own).  One CTA.
 __global__ void collect_units_kernel(const uint32_t *__restrict__ flags, int64_t U,
@@ -650,6 +675,41 @@ cudaError_t launch_colsum_keys(const TensorDesc &K, const TensorDesc &Q, const G
                                                                              raw, units);
     }
     return cudaGetLastError();
+}
+
+cudaError_t launch_recompute_units(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                                   float2 *partial, float *lse2, float *raw, const uint32_t *list,
+                                   cudaStream_t stream)
+{
+    int dev = 0, sms = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err == cudaSuccess)
+        err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess)
+        return err;
+    const int64_t blocks = g.U < sms ? g.U : sms;
+    const int rows_pad = (g.R + 7) & ~7;
+    const int bucket = max_ntw_bucket(rows_pad);
+    if (g.d == 128) {
+        const size_t smem = (size_t)(rows_pad + 2 * kTileKeys) * Pad<128>::kStride * 2;
+        DGE_DISPATCH_NTW(bucket, 128, recompute_units_kernel,
+                         err = prepare(k, smem);
+                         if (err == cudaSuccess) {
+                             k<<<(unsigned)blocks, kThreads, smem, stream>>>(K, Q, g, partial,
+                                                                             lse2, raw, list);
+                             err = cudaGetLastError();
+                         })
+    } else {
+        const size_t smem = (size_t)(rows_pad + 2 * kTileKeys) * Pad<64>::kStride * 2;
+        DGE_DISPATCH_NTW(bucket, 64, recompute_units_kernel,
+                         err = prepare(k, smem);
+                         if (err == cudaSuccess) {
+                             k<<<(unsigned)blocks, kThreads, smem, stream>>>(K, Q, g, partial,
+                                                                             lse2, raw, list);
+                             err = cudaGetLastError();
+                         })
+    }
+    return err;
 }
 
 cudaError_t launch_collect_units(const uint32_t *flags, int64_t U, uint32_t *units,

@@ -88,10 +88,12 @@ struct TcArgs {
     float *lse2;       // [U][R]
     float *raw;        // [U][P] (nrb == 1)
     unsigned long long *raw_fx;  // [U][P] fixed point, 2^-40 units (nrb > 1): row blocks add
-    uint32_t *count;   // [U]
-    uint32_t *ready;   // [U]
+    uint32_t *count;   // [U*nrb] phase-1 chunks counted in, per sub-unit
+    uint32_t *ready;   // [U] 2 = the unit left fp32's range (recomputed afterwards)
+    uint32_t *list;    // [1 + U] units to recompute: count, then ids
     uint32_t *status;
     unsigned long long timeout_ns;
+    int count_extra;   // chunks a unit's count must exceed nchunks by (0; > 0 only in tests)
     unsigned long long *trace;  // see dge_trace_set; nullptr = off
     int trace_cta;
 };
@@ -570,7 +572,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             // Bounded spin of one lane until every chunk of unit u is counted.
             auto spin_count = [&](const uint32_t *p) -> bool {
                 const uint64_t t0 = ptx::globaltimer();
-                while (ptx::ld_acquire_u32(p) < (uint32_t)a.nchunks) {
+                const uint32_t need = (uint32_t)(a.nchunks + a.count_extra);
+                while (ptx::ld_acquire_u32(p) < need) {
                     __nanosleep(64);
                     if (flag[kFlagAbort] || *(volatile uint32_t *)a.status != 0) {
                         flag[kFlagAbort] = 1;
@@ -668,8 +671,13 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 __syncwarp();
                 if (lane == 0) {
                     sm.sLbad[lb] = (!got || bad || flag[kFlagAbort]) ? 1 : 0;
-                    if (got && bad)
-                        a.ready[T.u] = kReadyBad;  // recomputed after the kernel
+                    if (got && bad) {
+                        // The unit (all of its row blocks) is recomputed after the kernel;
+                        // the first CTA to flag it lists it.
+                        const int64_t unit = T.u / a.nrb;
+                        if (atomicExch(&a.ready[unit], kReadyBad) != kReadyBad)
+                            a.list[1 + atomicAdd(a.list, 1u)] = (uint32_t)unit;
+                    }
                     trace_at<kTr>(a, kTrTimeline, 4 * (p2c - 1) + 3);
                     ptx::mbar_arrive(&sm.bar[kBarLseFull + lb]);
                 }
@@ -976,6 +984,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
 
 unsigned long long *g_trace = nullptr;
 int g_trace_cta = 0;
+unsigned long long g_wait_limit_ns = tc::kDefaultWaitLimitNs;
+int g_count_extra = 0;
 
 }  // namespace
 
@@ -1101,6 +1111,17 @@ void tc_set_trace(unsigned long long *buffer, int cta)
 {
     g_trace = buffer;
     g_trace_cta = cta;
+}
+
+void tc_set_waits(unsigned long long limit_ns, int count_extra)
+{
+    g_wait_limit_ns = limit_ns ? limit_ns : tc::kDefaultWaitLimitNs;
+    g_count_extra = count_extra;
+}
+
+unsigned long long tc_wait_limit_ns()
+{
+    return g_wait_limit_ns;
 }
 
 // Query heads per sub-unit: the most heads of a KV group (a divisor of G) whose stacked rows
@@ -1234,8 +1255,10 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.raw_fx = plan.nrb > 1 ? buf.raw_fx : nullptr;
     a.count = buf.count;
     a.ready = buf.ready;
+    a.list = buf.list;
     a.status = buf.status;
-    a.timeout_ns = 4000000000ull;
+    a.timeout_ns = g_wait_limit_ns;
+    a.count_extra = a.lse_in ? 0 : g_count_extra;
     a.trace = g_trace;
     a.trace_cta = g_trace_cta;
 

@@ -13,6 +13,9 @@ namespace tc {
 // Slot 0 of a kernel's shared flag block: set once the CTA has aborted.
 constexpr int kFlagAbort = 0;
 
+// Bound of every device-side wait of the tcgen05 kernels unless a test shortens it.
+constexpr unsigned long long kDefaultWaitLimitNs = 4000000000ull;
+
 // Bounded wait on an mbarrier phase.  Returns false when the CTA has aborted or the wait
 // outlived `timeout_ns` (then it aborts the CTA and records DGE_ERR_DEVICE_TIMEOUT).
 __device__ inline bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *flag,

@@ -42,6 +42,39 @@ def test_library_exports_every_declared_symbol(lib):
         assert name in B._SIGS, f"binding lacks {name}"
 
 
+def declared_signature(name):
+    """Parameter names of `name` as include/dge.h declares it."""
+    text = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    m = re.search(r"\b" + name + r"\s*\(([^)]*)\)\s*;", text)
+    assert m, name
+    params = [x.strip() for x in m.group(1).split(",") if x.strip() and x.strip() != "void"]
+    return [re.findall(r"(\w+)\s*$", x)[0] for x in params]
+
+
+# The boundary's calls with their parameters.  The scope table's boundary row lists
+# dge_select(p, scores, idx, ws, ws_bytes, stream) and dge_compact(p, idx, K, V, Kc, Vc,
+# stream); the library departs from it in two places, on purpose: dge_select takes no
+# workspace (the selection needs no device scratch and reports no device status), and
+# dge_compact takes an optional workspace whose status word receives out-of-range index
+# reports (NULL skips them).  Every other call matches the table.
+BOUNDARY = {
+    "dge_workspace_size": ["p", "bytes"],
+    "dge_score": ["p", "bufs", "ws", "ws_bytes", "stream"],
+    "dge_select": ["p", "scores", "idx", "stream"],
+    "dge_compact": ["p", "idx", "K", "V", "Kc", "Vc", "ws", "stream"],
+    "dge_evict": ["p", "bufs", "ws", "ws_bytes", "stream"],
+    "dge_pyramid_budgets": ["B", "w", "L", "out"],
+    "dge_get_device_status": ["ws", "stream"],
+    "dge_status_string": ["code"],
+}
+
+
+@pytest.mark.parametrize("name", sorted(BOUNDARY))
+def test_boundary_signatures(name):
+    assert declared_signature(name) == BOUNDARY[name]
+    assert len(B._SIGS[name]) == len(BOUNDARY[name])
+
+
 def test_struct_layout_matches_c():
     # int32 x6, int64, int32 x5, float, int32, pointer
     assert ctypes.sizeof(B.dge_problem) == 72

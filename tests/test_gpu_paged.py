@@ -204,3 +204,27 @@ def test_consecutive_pages(name, page_size, order):
     torch.cuda.synchronize()
     for k in ("idx", "Kc", "Vc", "scores"):
         assert torch.equal(got[k], ref[k]), k
+
+
+# --- paged runs against the oracle -------------------------------------------------------
+# The equality checks above tie a paged run to the contiguous run; these tie it to the fp64
+# oracle directly (scores, kept sets, gathered rows), so that a fault shared by both layouts,
+# or one only the paged producer has (per-page boxes, page clamping), cannot hide.
+
+@pytest.mark.parametrize("page_size", [16, 128])
+@pytest.mark.parametrize("name", ["c2_small", "c5_small", "c4_small", "slm_small"])
+def test_paged_evict_matches_oracle(name, page_size):
+    import oracle
+    from parity import compare_unit, oracle_units, unit_list
+    oracle.build()
+    wl = CASES[name]
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    want = wl.variant != inputs.STREAMING
+    K, V, pg = _paged(tens, page_size, seed=11 + page_size)
+    got = api.evict(p, K, V, _q(wl, tens), want_scores=want, paging=pg)
+    torch.cuda.synchronize()
+    units = unit_list(wl)
+    refs = oracle_units(wl, tens, units)
+    for (l, b, h) in units:
+        compare_unit(wl, got, tens, l, b, h, ref=refs[(l, b, h)])
