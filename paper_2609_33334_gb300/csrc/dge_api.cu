@@ -120,9 +120,9 @@ struct Plan {
     int chunk_keys = 0;      // phase-1 key chunk
     int nchunks = 0;
     TcPlan tc = {};          // tensor-core path decomposition (SCORED only)
-    size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, off_count = 0,
+    size_t off_partial = 0, off_lse = 0, off_raw = 0, off_pooled = 0, off_claim = 0, off_count = 0,
            off_ready = 0, off_rawfx = 0, off_units = 0, off_rpart = 0, ws_bytes = 0;
-    size_t flags_clear = 0;  // bytes from off_count that a tensor-core scoring call zeroes
+    size_t flags_clear = 0;  // bytes from off_claim that a tensor-core scoring call zeroes
 };
 
 constexpr int kScoredChunkKeys = 2048;
@@ -236,7 +236,7 @@ int make_plan(const dge_problem *p, Plan &plan)
             plan.tc = tc_plan(g);
             nrb = plan.tc.nrb;
             const size_t tc_bytes =
-                (size_t)g.U * nrb * plan.tc.r4 * plan.tc.nchunks * sizeof(float);
+                (size_t)g.U * nrb * plan.tc.r4 * plan.tc.nparts * sizeof(float);
             if (tc_bytes > part_bytes)
                 part_bytes = tc_bytes;
         }
@@ -249,13 +249,15 @@ int make_plan(const dge_problem *p, Plan &plan)
         plan.off_pooled = off;
         if (g.pool != DGE_POOL_NONE)
             off = align256(off + (size_t)g.U * g.P * sizeof(float));
-        // Flags, one region: chunk counters [U*nrb] (tensor-core path), per-unit range flags
-        // [U], then the list of units to recompute ([0] = count, [1 ..] = ids).  The counters,
-        // the flags and the list count are zeroed with one memset before a scoring launch.
-        plan.off_count = off;
-        plan.off_ready = off + (size_t)g.U * nrb * sizeof(uint32_t);
+        // Flags, one region: the task claim counter (tensor-core path; 16 bytes), chunk
+        // counters [U*nrb], per-unit range flags [U], then the list of units to recompute
+        // ([0] = count, [1 ..] = ids).  Everything up to the list count is zeroed with one
+        // memset before a scoring launch.
+        plan.off_claim = off;
+        plan.off_count = off + 16;
+        plan.off_ready = plan.off_count + (size_t)g.U * nrb * sizeof(uint32_t);
         plan.off_units = plan.off_ready + (size_t)g.U * sizeof(uint32_t);
-        plan.flags_clear = plan.off_units + sizeof(uint32_t) - plan.off_count;
+        plan.flags_clear = plan.off_units + sizeof(uint32_t) - plan.off_claim;
         off = align256(plan.off_units + (size_t)(g.U + 1) * sizeof(uint32_t));
         if (nrb > 1) {
             // Row blocks of one unit add their column sums in fixed point (exact, so the
@@ -404,7 +406,7 @@ int run_h2o_tc(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void 
                launch_colsum_keys(K, Q, g, lse2, raw, stream, units));
     if (lse_out)
         DGE_LAUNCH("lse_export", stream,
-                   launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
+                   launch_lse_export(nullptr, 0, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
                                      stream));
     return DGE_OK;
 }
@@ -429,6 +431,8 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
             tb.ready = nullptr;
             tb.status = static_cast<uint32_t *>(ws);
             tb.lse_in = lse_in;
+            tb.claim = ws_at<uint32_t>(ws, plan.off_claim);
+            DGE_CHECK_CUDA(cudaMemsetAsync(tb.claim, 0, sizeof(uint32_t), stream), "claim clear");
             unsigned long long *raw_fx = nullptr;
             if (plan.tc.nrb > 1) {
                 raw_fx = ws_at<unsigned long long>(ws, plan.off_rawfx);
@@ -461,10 +465,11 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
         return DGE_OK;
     }
     if (g.variant == DGE_VARIANT_SCORED && want_tc(g)) {
-        DGE_CHECK_CUDA(cudaMemsetAsync(ws_at<uint8_t>(ws, plan.off_count), 0, plan.flags_clear,
+        DGE_CHECK_CUDA(cudaMemsetAsync(ws_at<uint8_t>(ws, plan.off_claim), 0, plan.flags_clear,
                                        stream),
                        "flag clear");
         TcBuffers tb;
+        tb.claim = ws_at<uint32_t>(ws, plan.off_claim);
         tb.part = reinterpret_cast<float *>(partial);
         tb.lse2 = lse2;
         tb.raw = raw;
@@ -480,6 +485,11 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
                            "sum clear");
             tb.raw_fx = raw_fx;
         }
+        // The observation rows' own positions (causally masked), as the last chunk-sum slot;
+        // the main kernel covers the keys every row sees.
+        DGE_LAUNCH("score_tail", stream,
+                   launch_tail_rows(K, Q, g, plan.tc.rows, nrb, tb.part, plan.tc.nparts,
+                                    plan.tc.nchunks, plan.tc.r4, stream));
         bool encoded = false;
         DGE_LAUNCH("score_tc", stream,
                    launch_score_tc(K, Q, g, plan.tc, tb, stream, &encoded));
@@ -494,7 +504,8 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
                                               raw, tb.list, stream));
             if (lse_out)
                 DGE_LAUNCH("lse_export", stream,
-                           launch_lse_export(tb.part, plan.tc.nchunks, plan.tc.r4, lse2,
+                           launch_lse_export(tb.part, plan.tc.nparts, plan.tc.p1_chunks,
+                                             plan.tc.r4, lse2,
                                              tb.ready, g.U, g.R, plan.tc.rows, lse_out, stream));
             return DGE_OK;
         }
@@ -516,7 +527,7 @@ int run_scoring(const Plan &plan, const TensorDesc &K, const TensorDesc &Q, void
                    launch_colsum_rows(K, Q, g, kScoredChunkKeys, lse2, raw, stream));
     if (lse_out)
         DGE_LAUNCH("lse_export", stream,
-                   launch_lse_export(nullptr, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
+                   launch_lse_export(nullptr, 0, 0, 0, lse2, nullptr, g.U, g.R, g.R, lse_out,
                                      stream));
     return DGE_OK;
 }

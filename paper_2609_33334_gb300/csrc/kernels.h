@@ -27,6 +27,12 @@ cudaError_t launch_colsum_rows(const TensorDesc &K, const TensorDesc &Q, const G
 // The units whose flag (flags[U]) equals kUnitRecompute into units[1 + U] (count first).
 cudaError_t launch_collect_units(const uint32_t *flags, int64_t U, uint32_t *units,
                                  cudaStream_t stream);
+// Tensor-core scoring: the row sums of every sub-unit over the observation rows' own
+// positions [n - m, n) (masked causally), into chunk-sum slot `slot` of
+// part[U*nrb][nparts][r4].
+cudaError_t launch_tail_rows(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                             int rows, int nrb, float *part, int nparts, int slot, int r4,
+                             cudaStream_t stream);
 // SCORED units of a device-side list (list[0] = count, then ids), each recomputed whole by
 // one CTA with running maxima: row normalisers into lse2 (partial: [U][R] float2 scratch),
 // then the column sums into raw.  A capped grid: an empty list costs one read per CTA.
@@ -37,6 +43,8 @@ cudaError_t launch_recompute_units(const TensorDesc &K, const TensorDesc &Q, con
 // Scoring on the tcgen05 path (score_tc.cu).
 struct TcPlan {
     int r_pad, nslab, chunk_keys, nchunks, kstages;
+    int p1_chunks;     // chunks with keys below n - m (phase 1 covers [0, n - m))
+    int nparts;        // chunk-sum slots per sub-unit: nchunks + 1 (slot nchunks: the tail)
     int r4;            // row stride of the chunk sums: rows rounded up to 4 (16-byte rows)
     int gsub = 1;      // query heads per sub-unit (row block)
     int nrb = 1;       // sub-units per unit: G / gsub
@@ -44,7 +52,7 @@ struct TcPlan {
     size_t smem;
 };
 struct TcBuffers {
-    float *part;       // [U*nrb][nchunks][r4] row sums of each key chunk
+    float *part;       // [U*nrb][nparts][r4] row sums of each key chunk, then of the tail
     float *lse2;       // [U][R]
     float *raw;        // [U][P]
     unsigned long long *raw_fx = nullptr;  // [U][P], nrb > 1: fixed-point sums (2^-40)
@@ -52,6 +60,7 @@ struct TcBuffers {
     uint32_t *ready = nullptr;  // [U], zero before the launch; 2 = recompute
     uint32_t *list = nullptr;   // [1 + U], list[0] zero before the launch: the units flagged 2
     uint32_t *status = nullptr;
+    uint32_t *claim = nullptr;  // task claim counter, zero before the launch
     const float *lse_in = nullptr;  // [U][R] supplied natural-log normalisers (one pass)
 };
 bool tc_supported(const Geometry &g);
@@ -97,9 +106,11 @@ cudaError_t launch_h2o_tc(int phase, const TensorDesc &K, const TensorDesc &Q, c
 cudaError_t launch_pool(const float *raw, float *out, int64_t U, int P, int pool, int kernel,
                         cudaStream_t stream);
 // Row normalisers: caller's natural-log [U][R] -> base-2 lse2; lse2 (or, on the tensor-core
-// path, its chunk sums part [U][nchunks][r4] for units with ready != 2) -> natural-log out.
+// path, its chunk sums part [U*nrb][nparts][r4] -- slots 0 .. p1_chunks-1, then the tail's slot
+// nparts-1, in that order -- for units with ready != 2) -> natural-log out.
 cudaError_t launch_lse_import(const float *lse_in, float *lse2, int64_t total, cudaStream_t stream);
-cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const float *lse2,
+cudaError_t launch_lse_export(const float *part, int nparts, int p1_chunks, int r4,
+                              const float *lse2,
                               const uint32_t *ready, int64_t U, int R, int rows, float *lse_out,
                               cudaStream_t stream);
 // Fixed-point (2^-40) column sums of row blocks -> float.

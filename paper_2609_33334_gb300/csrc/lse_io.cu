@@ -26,7 +26,8 @@ __global__ void lse_import_kernel(const float *__restrict__ in, float *__restric
 // order, as that kernel merges them; row r of unit u is row r % rows of sub-unit
 // u * (R / rows) + r / rows) unless the unit was recomputed (ready == 2) or there are no chunk
 // sums (warp-level path), then from lse2.
-__global__ void lse_export_kernel(const float *__restrict__ part, int nchunks, int r4,
+__global__ void lse_export_kernel(const float *__restrict__ part, int nparts, int p1_chunks,
+                                  int r4,
                                   const float *__restrict__ lse2,
                                   const uint32_t *__restrict__ ready, int64_t U, int R, int rows,
                                   float *__restrict__ out)
@@ -40,9 +41,10 @@ __global__ void lse_export_kernel(const float *__restrict__ part, int nchunks, i
         if (part && !(ready && ready[u] == 2)) {
             float Z = 0.f;
             const int64_t sub = u * (R / rows) + r / rows;
-            const float *pu = part + sub * (int64_t)nchunks * r4 + r % rows;
-            for (int c = 0; c < nchunks; ++c)
+            const float *pu = part + sub * (int64_t)nparts * r4 + r % rows;
+            for (int c = 0; c < p1_chunks; ++c)
                 Z += pu[(int64_t)c * r4];
+            Z += pu[(int64_t)(nparts - 1) * r4];   // the tail, added last as the kernel does
             l2 = log2f(Z);
         } else {
             l2 = lse2[i];
@@ -74,11 +76,12 @@ cudaError_t launch_lse_import(const float *lse_in, float *lse2, int64_t total, c
     return cudaGetLastError();
 }
 
-cudaError_t launch_lse_export(const float *part, int nchunks, int r4, const float *lse2,
+cudaError_t launch_lse_export(const float *part, int nparts, int p1_chunks, int r4,
+                              const float *lse2,
                               const uint32_t *ready, int64_t U, int R, int rows, float *lse_out,
                               cudaStream_t stream)
 {
-    lse_export_kernel<<<blocks_for(U * (int64_t)R), 256, 0, stream>>>(part, nchunks, r4, lse2,
+    lse_export_kernel<<<blocks_for(U * (int64_t)R), 256, 0, stream>>>(part, nparts, p1_chunks, r4, lse2,
                                                                        ready, U, R, rows, lse_out);
     return cudaGetLastError();
 }

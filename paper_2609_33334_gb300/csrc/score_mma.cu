@@ -528,6 +528,89 @@ recompute_units_kernel(TensorDesc K, TensorDesc Q, Geometry g, float2 *__restric
     }
 }
 
+// Row sums over the observation rows' own positions, for the tensor-core scoring, whose main
+// kernel covers only the keys every row sees ([0, n - m)): sub-unit s = u * nrb + rb holds
+// rows rb * rows .. of unit u; row r sits at n - m + r % m and sees the keys n - m .. n - m +
+// r % m.  z_r = sum of 2^{x_rj} over them, in fp32 with no running maximum (the tensor-core
+// kernel's sums are plain too; its range check covers these), written to chunk-sum slot `slot`
+// of the sub-unit: part[(s * nparts + slot) * r4 + r].
+template <int D, int MAX_NTW>
+__global__ void __launch_bounds__(kThreads)
+tail_rows_kernel(TensorDesc K, TensorDesc Q, Geometry g, int rows, int nrb,
+                 float *__restrict__ part, int nparts, int slot, int r4)
+{
+    extern __shared__ __align__(16) uint8_t smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int gq = lane >> 2, tq = lane & 3;
+    const int rows_pad = (rows + 7) & ~7;
+    const int NT = rows_pad / 8;
+    const int first = g.n - g.m;
+    __nv_bfloat16 *sQ = reinterpret_cast<__nv_bfloat16 *>(smem);
+    __nv_bfloat16 *sK = sQ + rows_pad * Pad<D>::kStride;
+    for (int64_t s = blockIdx.x; s < g.U * nrb; s += gridDim.x) {
+        const int64_t u = s / nrb;
+        const int rb = (int)(s % nrb);
+        int l, bb, h;
+        unit_coords(g, u, l, bb, h);
+        stage_rows<D>(sQ, Q, g, l, bb, h, rb * rows, rows, rows_pad, g.m);
+        float z[MAX_NTW][2];
+        int lim[MAX_NTW][2];
+#pragma unroll
+        for (int i = 0; i < MAX_NTW; ++i)
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                const int nt = warp + 8 * i;
+                const int r = nt * 8 + 2 * tq + c;
+                z[i][c] = 0.f;
+                lim[i][c] = (nt < NT && r < rows) ? first + r % g.m : -1;
+            }
+        for (int k0 = first; k0 < g.n; k0 += kTileKeys) {
+            stage_keys<D, kTileKeys>(sK, K, l, bb, h, k0, g.n);
+            cp_async_commit();
+            cp_async_wait<0>();
+            __syncthreads();
+#pragma unroll 1
+            for (int mt = 0; mt < kTileKeys / 16; ++mt) {
+                if (k0 + mt * 16 >= g.n)
+                    break;
+                uint32_t a[D / 16][4];
+                load_a<D>(a, sK, mt, lane);
+                const int key0 = k0 + mt * 16 + gq, key1 = key0 + 8;
+#pragma unroll
+                for (int i = 0; i < MAX_NTW; ++i) {
+                    const int nt = warp + 8 * i;
+                    if (nt < NT) {
+                        float acc[4];
+                        tile_product<D>(acc, a, sQ, nt, lane);
+#pragma unroll
+                        for (int c = 0; c < 2; ++c) {
+                            const float ea = key0 <= lim[i][c] ? ex2(acc[c] * g.scale_log2) : 0.f;
+                            const float eb = key1 <= lim[i][c] ? ex2(acc[2 + c] * g.scale_log2)
+                                                               : 0.f;
+                            z[i][c] += ea + eb;
+                        }
+                    }
+                }
+            }
+            __syncthreads();
+        }
+        // The 8 lanes that share each row (lane bits 2..4), in a fixed order.
+#pragma unroll
+        for (int i = 0; i < MAX_NTW; ++i)
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                float v = z[i][c];
+                v += __shfl_xor_sync(0xffffffffu, v, 4);
+                v += __shfl_xor_sync(0xffffffffu, v, 8);
+                v += __shfl_xor_sync(0xffffffffu, v, 16);
+                const int nt = warp + 8 * i;
+                const int r = nt * 8 + 2 * tq + c;
+                if (gq == 0 && nt < NT && r < rows)
+                    part[(s * nparts + slot) * r4 + r] = v;
+            }
+    }
+}
+
 // The units flagged kUnitRecompute, as a list (units[0] = count, then the ids in any order:
 // every unit is recomputed on its own).  One CTA.
 __global__ void collect_units_kernel(const uint32_t *__restrict__ flags, int64_t U,
@@ -706,6 +789,42 @@ cudaError_t launch_recompute_units(const TensorDesc &K, const TensorDesc &Q, con
                          if (err == cudaSuccess) {
                              k<<<(unsigned)blocks, kThreads, smem, stream>>>(K, Q, g, partial,
                                                                              lse2, raw, list);
+                             err = cudaGetLastError();
+                         })
+    }
+    return err;
+}
+
+cudaError_t launch_tail_rows(const TensorDesc &K, const TensorDesc &Q, const Geometry &g,
+                             int rows, int nrb, float *part, int nparts, int slot, int r4,
+                             cudaStream_t stream)
+{
+    int dev = 0, sms = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err == cudaSuccess)
+        err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess)
+        return err;
+    const int64_t subs = g.U * nrb;
+    const int64_t blocks = subs < (int64_t)sms * 8 ? subs : (int64_t)sms * 8;
+    const int rows_pad = (rows + 7) & ~7;
+    const int bucket = max_ntw_bucket(rows_pad);
+    if (g.d == 128) {
+        const size_t smem = (size_t)(rows_pad + kTileKeys) * Pad<128>::kStride * 2;
+        DGE_DISPATCH_NTW(bucket, 128, tail_rows_kernel,
+                         err = prepare(k, smem);
+                         if (err == cudaSuccess) {
+                             k<<<(unsigned)blocks, kThreads, smem, stream>>>(
+                                 K, Q, g, rows, nrb, part, nparts, slot, r4);
+                             err = cudaGetLastError();
+                         })
+    } else {
+        const size_t smem = (size_t)(rows_pad + kTileKeys) * Pad<64>::kStride * 2;
+        DGE_DISPATCH_NTW(bucket, 64, tail_rows_kernel,
+                         err = prepare(k, smem);
+                         if (err == cudaSuccess) {
+                             k<<<(unsigned)blocks, kThreads, smem, stream>>>(
+                                 K, Q, g, rows, nrb, part, nparts, slot, r4);
                              err = cudaGetLastError();
                          })
     }

@@ -16,13 +16,16 @@
 //               tasks;
 //   warps 4-15  epilogue: three warpgroups, each thread one key (TMEM lane),
 //               each warpgroup a third of the row columns.
-// Work items are (unit, key chunk).  Step t of CTA s runs phase 1 of item
-// t*S + s (per-row sums 2^x over the chunk) and then phase 2 of item
-// (t-1)*S + s - (nchunks-1) (2^{x - lse} summed over rows per key), so phase 2
-// re-reads a chunk streamed about one step earlier while it is still in L2, and
-// only needs units whose every chunk finished phase 1 in an earlier step.  Row sums use no
-// running maximum: fp32 holds 2^x for |x| < 126, and a unit whose sums leave
-// [2^-60, 2^126) is flagged (ready = 2) and recomputed by the warp-level path.
+// Work items are (unit, key chunk).  Tasks -- phase 1 of an item (per-row sums 2^x over the
+// chunk) or phase 2 (2^{x - lse} summed over rows per key) -- form one sequence in which
+// phase 1 of item lag + j and phase 2 of item j alternate; each CTA's producer claims the
+// next task from a global counter when it needs one, and hands it to the other roles
+// through a ring in shared memory.  Claiming in sequence order keeps the CTAs together (a
+// slow CTA claims fewer tasks, so no CTA falls behind the others), so phase 2 re-reads a
+// chunk about `lag` items after its phase-1 read, while it is still in L2, and a task only
+// ever waits for tasks claimed before it.  Row sums use no running maximum: fp32 holds 2^x
+// for |x| < 126, and a unit whose sums leave [2^-60, 2^126) is flagged (ready = 2) and
+// recomputed by the warp-level path.
 //
 // Every wait is bounded: on expiry the CTA records DGE_ERR_DEVICE_TIMEOUT in the
 // status word, stops issuing work, waits (bounded) for its own copies and MMAs,
@@ -30,6 +33,8 @@
 #include <cuda.h>
 #include <math.h>
 #include <string.h>
+
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -61,9 +66,23 @@ constexpr uint32_t kReadyBad = 2;          // unit left fp32's range: recomputed
 // Barrier slots.
 constexpr int kBarKFull = 0, kBarKEmpty = 4, kBarQFull = 8, kBarQEmpty = 10, kBarAccFull = 12,
               kBarAccEmpty = 15, kBarDrain = 18, kBarRedFull = 19, kBarRedEmpty = 21,
-              kBarLseFull = 23, kBarLseEmpty = 25, kBarStage = 27, kBarXch = 28, kNumBars = 40;
+              kBarLseFull = 23, kBarLseEmpty = 25, kBarStage = 27, kBarXch = 28,
+              kBarRingFull = 40, kBarRingEmpty = 48, kNumBars = 56;
+constexpr int kRing = 8;                  // claimed tasks handed from the producer to the others
+// Lag of the claim sequence in tenths of the grid (see launch_score_tc) and the key tiles of a
+// task of whole units (see tc_plan).
+#ifndef DGE_TC_LAG_GRID_X10
+#define DGE_TC_LAG_GRID_X10 15
+#endif
+#ifndef DGE_TC_CHUNK_TILES
+#define DGE_TC_CHUNK_TILES 48
+#endif
+constexpr int kLagGridX10 = DGE_TC_LAG_GRID_X10;
+constexpr int kChunkTiles = DGE_TC_CHUNK_TILES;
+// Arrivals that free a ring slot: the MMA warp, the two coordinator warps, the epilogue warps.
+constexpr int kRingConsumers = 3 + 12;
 constexpr int kStageBytes = 12288;        // chunk sums of a unit, staged for the lse merge
-constexpr int kCtrlBytes = 400;            // barriers, TMEM address, flags (16-byte multiple)
+constexpr int kCtrlBytes = 640;            // barriers, TMEM address, flags, ring (16-byte multiple)
 constexpr int kRowsPerLane = 5;           // rows of the lse merge per lane (R <= 160)
 // Flag slots (ints): abort, then the parity of the last arm of every key stage, query
 // buffer and the staging buffer (-1 = never armed) for the drain.
@@ -77,13 +96,16 @@ struct TcArgs {
     int r_pad, r4, nslab, kstages;
     int acc_stride;    // TMEM columns between accumulator buffers
     int unit_tiles, nchunks;   // key tiles of a unit; chunk c = tiles [c*T/nc, (c+1)*T/nc)
+    int p1_chunks;     // chunks with phase-1 keys (the first ones: they start below n - m)
+    int nparts;        // chunk-sum slots per sub-unit: nchunks, then the tail's (slot nchunks)
     int64_t items;
-    int64_t lag;       // extra items between an item's phase-1 and phase-2 tasks
+    int64_t lag;       // items between an item's phase-1 and phase-2 tasks (>= nchunks - 1)
+    int64_t total;     // tasks in the claim sequence
+    uint32_t *claim;   // claim counter, zero before the launch
     const float *lse_in;  // [U][R] natural-log row normalisers supplied by the caller: then
                           // there is no phase 1 and phase 2 of item t*S + s runs in step t
     int ng[kEpiWG];    // 16-column groups of each epilogue warpgroup
     int gbase[kEpiWG]; // first group of each epilogue warpgroup
-    int64_t steps;
     float *part;       // [U][nchunks][r4]
     float *lse2;       // [U][R]
     float *raw;        // [U][P] (nrb == 1)
@@ -138,33 +160,41 @@ struct Task {
     int chunk, k_lo, k_hi, ntiles;
 };
 
-// Task j (0: phase 1, 1: phase 2) of step t for this CTA: phase 1 of item t*S + s, phase 2
-// of item (t-1)*S + s - lag.  With lag = nchunks - 1, every unit a phase-2 task needs was
-// completed by phase-1 tasks of earlier steps (a unit's chunks may straddle two steps).
-// False when there is none (or it covers no keys).
-__device__ __forceinline__ bool get_task(const TcArgs &a, int64_t t, int j, Task &T)
+// Task p of the claim sequence.  Items are item = u * nchunks + chunk.  Positions 0 .. lag-1
+// are phase 1 of items 0 .. lag-1; then phase 1 of item lag + j and phase 2 of item j
+// alternate; the last lag positions are phase 2 of the last lag items.  A unit's last chunk
+// is at most nchunks - 1 items after any of its chunks, so with lag >= nchunks - 1 phase 2 of
+// every chunk of a unit comes after phase 1 of all of them.  With normalisers supplied
+// (lse_in) the sequence is phase 2 of every item in order.  False when p is past the end or
+// the task covers no keys.
+__device__ __forceinline__ bool task_at(const TcArgs &a, int64_t p, Task &T)
 {
-    const int64_t S = gridDim.x, s = blockIdx.x;
     int64_t item;
     if (a.lse_in) {
-        if (j == 0)
-            return false;
-        item = t * S + s;
+        item = p;
         T.phase = 2;
-    } else if (j == 0) {
-        item = t * S + s;
+    } else if (p < a.lag) {
+        item = p;
         T.phase = 1;
     } else {
-        item = (t - 1) * S + s - a.lag;
-        T.phase = 2;
+        const int64_t q = p - a.lag, mid = 2 * (a.items - a.lag);
+        if (q < mid) {
+            item = (q & 1) ? (q >> 1) : a.lag + (q >> 1);
+            T.phase = (q & 1) ? 2 : 1;
+        } else {
+            item = a.items - a.lag + (q - mid);
+            T.phase = 2;
+        }
     }
-    if (item < 0 || item >= a.items)
+    if (p < 0 || p >= a.total || item < 0 || item >= a.items)
         return false;
     T.u = item / a.nchunks;
     T.chunk = (int)(item % a.nchunks);
     T.k_lo = (int)((int64_t)T.chunk * a.unit_tiles / a.nchunks) * kTile;
     const int k_end = (int)((int64_t)(T.chunk + 1) * a.unit_tiles / a.nchunks) * kTile;
-    const int end = T.phase == 1 ? a.g.n : a.g.P;
+    // Phase 1 covers the keys every observation row sees, [0, n - m); the rows' own positions
+    // [n - m, n) are added by the tail kernel (masked there).  Phase 2 covers [0, P), P <= n - m.
+    const int end = T.phase == 1 ? a.g.n - a.g.m : a.g.P;
     T.k_hi = min(k_end, end);
     if (T.k_lo >= T.k_hi)
         return false;
@@ -179,6 +209,7 @@ struct Smem {
     uint64_t *bar;       // [kNumBars]
     uint32_t *tmem;      // allocation result
     int *flag;           // [16]
+    volatile int64_t *ring;  // [kRing] claimed task positions (-1: no more tasks)
     float *sL;           // [2][256] -lse of the rows of a phase-2 task (padding: -inf)
     float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
@@ -213,7 +244,8 @@ __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int ks
     s.bar = reinterpret_cast<uint64_t *>(raw + off);
     s.tmem = reinterpret_cast<uint32_t *>(raw + off + kNumBars * 8);
     s.flag = reinterpret_cast<int *>(raw + off + kNumBars * 8 + 16);
-    static_assert(kNumBars * 8 + 16 + 64 <= kCtrlBytes, "control block");
+    s.ring = reinterpret_cast<int64_t *>(raw + off + kNumBars * 8 + 16 + 64);
+    static_assert(kNumBars * 8 + 16 + 64 + kRing * 8 <= kCtrlBytes, "control block");
     off += kCtrlBytes;
     s.sL = reinterpret_cast<float *>(raw + off);  // 16-byte aligned: read as float4
     off += 2 * 256 * 4;
@@ -238,65 +270,63 @@ using tc::drain_bar;
 using tc::transpose_sum16;
 using tc::transpose_sum32;
 
-// Visibility of the 16 columns cb .. cb+15 to `key` on tiles that reach the observation
-// rows' own positions: row r sits at first_causal + r % m and sees keys up to there.
-__device__ __forceinline__ uint32_t causal_mask(int key, int first_causal, int cb, int m)
-{
-    uint32_t mask = 0;
-#pragma unroll
-    for (int c = 0; c < 16; ++c)
-        mask |= (key <= first_causal + (cb + c) % m ? 1u : 0u) << c;
-    return mask;
-}
 
-// Phase 1 for one 16-column group: z[c] += 2^{x_c} (masked columns add nothing).
-__device__ __forceinline__ void rows_add(float (&z)[16], const float (&v)[16], float s2, bool valid,
-                                         bool causal, int key, int first_causal, int cb, int m)
+// Phase 1 for one 16-column group: z[c] += 2^{x_c} (every row sees every key of phase 1).
+// A group with exactly 8 query rows (cvalid == 8, the last group of 136 stacked rows) skips
+// the exponentials of its 8 padding columns; any other group computes all 16.
+__device__ __forceinline__ void rows_add(float (&z)[16], const float (&w)[16], float s2, bool valid,
+                                         int cvalid)
 {
     if (!valid)
         return;
-    if (!causal) {
-        const float2 sc = make_float2(s2, s2);
+    const float2 sc = make_float2(s2, s2);
+    // Fully unrolled either way (a per-pair bound check would serialise the exponentials).
+    auto pairs = [&](auto npairs) {
 #pragma unroll
-        for (int c = 0; c < 16; c += 2) {
-            const float2 x = __fmul2_rn(make_float2(v[c], v[c + 1]), sc);
+        for (int c = 0; c < 2 * decltype(npairs)::value; c += 2) {
+            const float2 x = __fmul2_rn(make_float2(w[c], w[c + 1]), sc);
             const float2 acc = __fadd2_rn(make_float2(z[c], z[c + 1]),
                                           make_float2(ex2(x.x), ex2(x.y)));
             z[c] = acc.x;
             z[c + 1] = acc.y;
         }
-    } else {
-        const uint32_t mask = causal_mask(key, first_causal, cb, m);
-#pragma unroll
-        for (int c = 0; c < 16; ++c) {
-            const float e = ex2(v[c] * s2);
-            z[c] += ((mask >> c) & 1u) ? e : 0.f;
-        }
-    }
+    };
+    if (cvalid == 8)
+        pairs(std::integral_constant<int, 4>());
+    else
+        pairs(std::integral_constant<int, 8>());
 }
 
 // Phase 2 for one 16-column group: adds 2^{x_c - lse_c} over the group's rows into the
-// pair accumulator.  nL holds -lse (padded columns: -inf).
-__device__ __forceinline__ void col_add(float2 &acc, const float (&v)[16], const float (&nL)[16],
-                                        float s2, bool causal, int key, int first_causal, int cb,
-                                        int m)
+// pair accumulator.  nL holds -lse (padded columns: -inf, so they add exactly 0; a group of
+// exactly 8 rows, cvalid == 8, skips its 8 padding columns).
+__device__ __forceinline__ void col_add(float2 &acc, const float (&w)[16], const float *nLs,
+                                        float s2, int cvalid)
 {
-    if (!causal) {
-        const float2 sc = make_float2(s2, s2);
+    // -lse of the group's 16 rows, from the task's staging buffer (the same 16 values for
+    // every lane: broadcast loads).
+    float nL[16];
 #pragma unroll
-        for (int c = 0; c < 16; c += 2) {
-            const float2 x = __ffma2_rn(make_float2(v[c], v[c + 1]), sc,
+    for (int i = 0; i < 4; ++i) {
+        const float4 q = reinterpret_cast<const float4 *>(nLs)[i];
+        nL[4 * i] = q.x;
+        nL[4 * i + 1] = q.y;
+        nL[4 * i + 2] = q.z;
+        nL[4 * i + 3] = q.w;
+    }
+    const float2 sc = make_float2(s2, s2);
+    auto pairs = [&](auto npairs) {
+#pragma unroll
+        for (int c = 0; c < 2 * decltype(npairs)::value; c += 2) {
+            const float2 x = __ffma2_rn(make_float2(w[c], w[c + 1]), sc,
                                         make_float2(nL[c], nL[c + 1]));
             acc = __fadd2_rn(acc, make_float2(ex2(x.x), ex2(x.y)));
         }
-    } else {
-        const uint32_t mask = causal_mask(key, first_causal, cb, m);
-#pragma unroll
-        for (int c = 0; c < 16; ++c) {
-            const float p = ex2(v[c] * s2 + nL[c]);
-            acc.x += ((mask >> c) & 1u) ? p : 0.f;
-        }
-    }
+    };
+    if (cvalid == 8)
+        pairs(std::integral_constant<int, 4>());
+    else
+        pairs(std::integral_constant<int, 8>());
 }
 
 // Runs f(gi, v) over this warp's lane quarter of 16-column groups gi = 0 .. ng-1 (ng <=
@@ -314,6 +344,8 @@ __device__ __forceinline__ void for_groups(uint32_t tbase, int ng, F &&f)
             f(gi, v);
         }
 }
+
+
 
 // kTr: with the cycle accounting and timelines of dge_trace_set (a separate build, so the
 // clock reads cost nothing when tracing is off).  kFx: units split into row blocks whose
@@ -362,6 +394,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         // warpgroup.
         for (int i = 0; i < kAccBufs * 4; ++i)
             ptx::mbar_init(&sm.bar[kBarXch + i], kEpiWG);
+        for (int i = 0; i < kRing; ++i) {
+            ptx::mbar_init(&sm.bar[kBarRingFull + i], 1);
+            ptx::mbar_init(&sm.bar[kBarRingEmpty + i], kRingConsumers);
+        }
         ptx::fence_mbar_init();
     }
     // Query rows R .. r_pad-1 are never written by TMA: zero them once so the padded
@@ -403,11 +439,27 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             long long cy_wq = 0, cy_wk = 0;
             const long long cy0 = tclock<kTr>();
             bool ok = true;
-            for (int64_t t = 0; ok && t <= a.steps; ++t)
-                for (int j = 0; ok && j < 2; ++j) {
+            // The next task this CTA takes is claimed while the current one's last tiles are
+            // issued, so the claim's round trip is hidden and the task is not held long.
+            uint32_t pending = atomicAdd(a.claim, 1u);
+            for (int k = 0; ok; ++k) {
                     Task T;
-                    if (!get_task(a, t, j, T))
-                        continue;
+                    int64_t p = -1;
+                    for (uint32_t c = pending; (int64_t)c < a.total; c = atomicAdd(a.claim, 1u))
+                        if (task_at(a, c, T)) {
+                            p = c;
+                            break;
+                        }
+                    const int slot = k % kRing;
+                    if (!wait_bar(&sm.bar[kBarRingEmpty + slot], (uint32_t)((k / kRing) & 1) ^ 1u,
+                                  flag, a)) {
+                        ok = false;
+                        break;
+                    }
+                    sm.ring[slot] = p;
+                    ptx::mbar_arrive(&sm.bar[kBarRingFull + slot]);
+                    if (p < 0)
+                        break;
                     int l, bb, h;
                     unit_coords(g, kFx ? T.u / a.nrb : T.u, l, bb, h);
 
@@ -432,6 +484,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     int w0 = 0;               // first key of the page-id window (paged caches)
                     const int *ids = sm.pages;
                     for (int tile = 0; tile < T.ntiles; ++tile) {
+                        if (tile == max(T.ntiles - 2, 0))
+                            pending = atomicAdd(a.claim, 1u);
                         if constexpr (kPaged) {
                             if (tile % tc::kPageWindowTiles == 0) {
                                 w0 = T.k_lo + tile * kTile;
@@ -474,11 +528,16 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             long long cy_wq = 0, cy_wk = 0, cy_wa = 0, cy_is = 0, cy_cm = 0;
             const long long cy0 = tclock<kTr>();
             bool ok = true;
-            for (int64_t t = 0; ok && t <= a.steps; ++t)
-                for (int j = 0; ok && j < 2; ++j) {
+            for (int k = 0; ok; ++k) {
+                    const int slot = k % kRing;
+                    if (!wait_bar(&sm.bar[kBarRingFull + slot], (uint32_t)((k / kRing) & 1), flag,
+                                  a))
+                        break;
+                    const int64_t p = sm.ring[slot];
+                    ptx::mbar_arrive(&sm.bar[kBarRingEmpty + slot]);
                     Task T;
-                    if (!get_task(a, t, j, T))
-                        continue;
+                    if (p < 0 || !task_at(a, p, T))
+                        break;
                     long long c0 = tclock<kTr>();
                     if (!wait_bar(&sm.bar[kBarQFull + qb], qph, flag, a)) {
                         ok = false;
@@ -558,8 +617,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         // every chunk of the task's unit is counted, brings the unit's chunk sums into
         // shared memory with bulk copies, adds them in chunk order (the same result in every
         // CTA that needs the unit) and stages -lse for the epilogue.  The two warps never
-        // wait on each other, and a phase-2 task of step t needs only phase-1 tasks of
-        // earlier steps, so the waits cannot form a cycle.
+        // wait on each other, and a phase-2 task needs only phase-1 tasks claimed before it,
+        // so the waits cannot form a cycle.
         bool dead = false;
         auto wait_w = [&](uint64_t *bar, uint32_t parity) {
             if (!dead) {
@@ -568,11 +627,23 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             }
             return !dead;
         };
+        // This CTA's k-th claimed task from the ring (the whole warp reads it; lane 0 frees
+        // the slot).  False at the end of the sequence or once the CTA is dead.
+        auto ring_task = [&](int k, Task &T) -> bool {
+            const int slot = k % kRing;
+            if (!wait_w(&sm.bar[kBarRingFull + slot], (uint32_t)((k / kRing) & 1)))
+                return false;
+            const int64_t p = sm.ring[slot];
+            __syncwarp();
+            if (lane == 0)
+                ptx::mbar_arrive(&sm.bar[kBarRingEmpty + slot]);
+            return p >= 0 && task_at(a, p, T);
+        };
         if (warp == 2) {
             // Bounded spin of one lane until every chunk of unit u is counted.
             auto spin_count = [&](const uint32_t *p) -> bool {
                 const uint64_t t0 = ptx::globaltimer();
-                const uint32_t need = (uint32_t)(a.nchunks + a.count_extra);
+                const uint32_t need = (uint32_t)(a.p1_chunks + a.count_extra);
                 while (ptx::ld_acquire_u32(p) < need) {
                     __nanosleep(64);
                     if (flag[kFlagAbort] || *(volatile uint32_t *)a.status != 0) {
@@ -590,9 +661,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             const int per_piece = kStageBytes / (a.r4 * 4);  // chunks per bulk copy
             uint32_t sph = 0;
             int p2c = 0;
-            for (int t = 0; t <= (int)a.steps; ++t) {
+            for (int k = 0;; ++k) {
                 Task T;
-                if (!get_task(a, t, 1, T))
+                if (!ring_task(k, T))
+                    break;
+                if (T.phase != 2)
                     continue;
                 const int lb = p2c & 1;
                 const uint32_t lph = (uint32_t)((p2c >> 1) & 1);
@@ -627,9 +700,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
 #pragma unroll
                 for (int i = 0; i < kRowsPerLane; ++i)
                     Z[i] = 0.f;
-                const float *src = a.part + T.u * a.nchunks * a.r4;
-                for (int c0 = 0; got && c0 < a.nchunks; c0 += per_piece) {
-                    const int nc = min(per_piece, a.nchunks - c0);
+                // Slots 0 .. p1_chunks-1 (chunk order), then the tail's slot nchunks; the
+                // slots in between belong to chunks with no phase-1 keys and are skipped.
+                const float *src = a.part + T.u * a.nparts * a.r4;
+                for (int c0 = 0; got && c0 < a.nparts; c0 += per_piece) {
+                    const int nc = min(per_piece, a.nparts - c0);
                     __syncwarp();
                     if (lane == 0) {
                         // The previous piece's reads (generic proxy) come before the copy.
@@ -644,13 +719,16 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         break;
                     }
                     sph ^= 1;
-                    for (int c = 0; c < nc; ++c)
+                    for (int c = 0; c < nc; ++c) {
+                        if (c0 + c >= a.p1_chunks && c0 + c < a.nchunks)
+                            continue;
 #pragma unroll
                         for (int i = 0; i < kRowsPerLane; ++i) {
                             const int r = lane + 32 * i;
                             if (r < a.rows)
                                 Z[i] += sm.stage[c * a.r4 + r];
                         }
+                    }
                 }
                 bool bad = false;
                 float *L = sm.sL + lb * 256;
@@ -684,9 +762,11 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             }
         } else {
             int p1c = 0;
-            for (int t = 0; t <= (int)a.steps; ++t) {
+            for (int k = 0;; ++k) {
                 Task T;
-                if (!get_task(a, t, 0, T))
+                if (!ring_task(k, T))
+                    break;
+                if (T.phase != 1)
                     continue;
                 const int rb = p1c & 1;
                 const uint32_t rph = (uint32_t)((p1c >> 1) & 1);
@@ -694,7 +774,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 const bool ok = wait_w(&sm.bar[kBarRedFull + rb], rph);
                 if (ok) {
                     constexpr int W = kMaxGroups * 16;
-                    float *dst = a.part + (T.u * a.nchunks + T.chunk) * a.r4;
+                    float *dst = a.part + (T.u * a.nparts + T.chunk) * a.r4;
                     for (int col = lane; col < a.rows; col += 32) {
                         int w = 0;
                         while (w + 1 < kEpiWG && col >= a.gbase[w + 1] * 16)
@@ -731,7 +811,6 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
         const int col_base = a.gbase[wg] * 16;
         const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
         const float s2 = g.scale_log2;
-        const int first_causal = g.n - g.m;      // keys from here on are not seen by every row
         int tc = 0;   // accumulator tiles consumed (buffer tc % 3, use tc / 3)
         int p1c = 0;  // phase-1 tasks (row-sum hand-off buffer p1c % 2)
         int p2c = 0;  // phase-2 tasks (-lse buffer p2c % 2)
@@ -771,11 +850,22 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             cy_rel += tclock<kTr>() - c0;
         };
 
-        for (int t = 0; t <= (int)a.steps; ++t)
-            for (int j = 0; j < 2; ++j) {
+        for (int k = 0;; ++k) {
                 Task T;
-                if (!get_task(a, t, j, T))
-                    continue;
+                {
+                    // This CTA's k-th claimed task (every epilogue warp frees the slot once).
+                    const int slot = k % kRing;
+                    if (!wait_uniform(&sm.bar[kBarRingFull + slot], (uint32_t)((k / kRing) & 1)))
+                        break;
+                    const int64_t p = sm.ring[slot];
+                    __syncwarp();
+                    if (lane == 0)
+                        ptx::mbar_arrive(&sm.bar[kBarRingEmpty + slot]);
+                    if (p < 0 || !task_at(a, p, T))
+                        break;
+                }
+                if (ew == 0 && lane == 0)
+                    trace_at<kTr>(a, kTrTimeline, 3072 + 4 * k);
                 if (T.phase == 1) {
                     // ---------------- phase 1: row sums over this chunk ----------------
                     float z[kMaxGroups][16];
@@ -790,24 +880,26 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         const int tile0 = T.k_lo + tile * kTile;
                         const int key = tile0 + kl;
                         const bool valid = key < T.k_hi;
-                        const bool causal = tile0 + kTile > first_causal;
                         if (acquire_acc(ab, aph)) {
                             // All of this warp's columns in one TMEM round trip.
                             const uint32_t tbase =
                                 tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
                             const long long c0 = tclock<kTr>();
-                            for_groups(tbase, ng, [&](int gi, const float(&v)[16]) {
+                            auto f1 = [&](int gi, const float(&v)[16]) {
 #pragma unroll
                                 for (int gj = 0; gj < kMaxGroups; ++gj)
                                     if (gj == gi)
-                                        rows_add(z[gj], v, s2, valid, causal, key, first_causal,
-                                                 col_base + gj * 16, g.m);
-                            });
+                                        rows_add(z[gj], v, s2, valid,
+                                                 a.rows - (col_base + gj * 16));
+                            };
+                            for_groups(tbase, ng, f1);
                             cy_math += tclock<kTr>() - c0;
                         }
                         release_acc(ab, 1u);
                     }
                     const long long c_end = tclock<kTr>();
+                    if (ew == 0 && lane == 0)
+                        trace_at<kTr>(a, kTrTimeline, 3072 + 4 * k + 1);
                     // Sums over this warp's 32 keys, handed to the coordinator warps through
                     // a double-buffered area (they add the warps in a fixed order).
                     const int rb = p1c & 1;
@@ -821,6 +913,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                                 transpose_sum16(z[gi], lane);
                         }
                     }
+                    if (ew == 0 && lane == 0)
+                        trace_at<kTr>(a, kTrTimeline, 3072 + 4 * k + 2);
                     if (wait_uniform(&sm.bar[kBarRedEmpty + rb], rph ^ 1)) {
                         float *red = sm.red + ((rb * kEpiWG + wg) * 4 + quarter) * (kMaxGroups * 16);
 #pragma unroll
@@ -835,6 +929,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         __syncwarp();
                         if (lane == 0)
                             ptx::mbar_arrive(&sm.bar[kBarRedFull + rb]);
+                        if (ew == 0 && lane == 0)
+                            trace_at<kTr>(a, kTrTimeline, 3072 + 4 * k + 3);
                     }
                     ++p1c;
                     cy_p1e += tclock<kTr>() - c_end;
@@ -848,34 +944,14 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     ++p2c;
                     if (ew == 0 && lane == 0)
                         trace_at<kTr>(a, kTrTimeline, 2048 + 2 * (p2c - 1));
-                    float nL[kMaxGroups][16];
+                    // -lse of this warpgroup's columns stays in the staging buffer for the
+                    // whole task (read per group with broadcast loads); the buffer is freed
+                    // after the task's last tile.
+                    const float *nLs = sm.sL + lb * 256 + col_base;
                     bool task_ok = false;
-                    if (wait_uniform(&sm.bar[kBarLseFull + lb], lph)) {
-                        const float4 *L4 =
-                            reinterpret_cast<const float4 *>(sm.sL + lb * 256 + col_base);
-#pragma unroll
-                        for (int gi = 0; gi < kMaxGroups; ++gi)
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const float4 q = gi < ng ? L4[gi * 4 + i]
-                                                         : make_float4(-INFINITY, -INFINITY,
-                                                                       -INFINITY, -INFINITY);
-                                nL[gi][4 * i] = q.x;
-                                nL[gi][4 * i + 1] = q.y;
-                                nL[gi][4 * i + 2] = q.z;
-                                nL[gi][4 * i + 3] = q.w;
-                            }
+                    const bool have_lse = wait_uniform(&sm.bar[kBarLseFull + lb], lph);
+                    if (have_lse)
                         task_ok = sm.sLbad[lb] == 0;
-                        __syncwarp();
-                        if (lane == 0)
-                            ptx::mbar_arrive(&sm.bar[kBarLseEmpty + lb]);
-                    } else {
-#pragma unroll
-                        for (int gi = 0; gi < kMaxGroups; ++gi)
-#pragma unroll
-                            for (int c = 0; c < 16; ++c)
-                                nL[gi][c] = -INFINITY;
-                    }
                     if (ew == 0 && lane == 0)
                         trace_at<kTr>(a, kTrTimeline, 2048 + 2 * (p2c - 1) + 1);
                     task_ok = task_ok && !dead;
@@ -890,19 +966,19 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
                         const int tile0 = T.k_lo + tile * kTile;
                         const int key = tile0 + kl;
-                        const bool causal = tile0 + kTile > first_causal;
                         float2 acc = make_float2(0.f, 0.f);
                         if (acquire_acc(ab, aph)) {
                             const uint32_t tbase =
                                 tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
                             const long long c0 = tclock<kTr>();
-                            for_groups(tbase, ng, [&](int gi, const float(&v)[16]) {
+                            auto f2 = [&](int gi, const float(&v)[16]) {
 #pragma unroll
                                 for (int gj = 0; gj < kMaxGroups; ++gj)
                                     if (gj == gi)
-                                        col_add(acc, v, nL[gj], s2, causal, key, first_causal,
-                                                col_base + gj * 16, g.m);
-                            });
+                                        col_add(acc, v, nLs + gj * 16, s2,
+                                                a.rows - (col_base + gj * 16));
+                            };
+                            for_groups(tbase, ng, f2);
                             cy_math2 += tclock<kTr>() - c0;
                         }
                         // The three warps of this lane quarter (one per warpgroup) leave their
@@ -948,6 +1024,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         cy_xch += tclock<kTr>() - cx;
                         release_acc(ab, 1u);
                     }
+                    // The -lse buffer is free for the coordinator's next-but-one task.
+                    __syncwarp();
+                    if (have_lse && lane == 0)
+                        ptx::mbar_arrive(&sm.bar[kBarLseEmpty + lb]);
                 }
             }
         if (ew == 0 && lane == 0) {
@@ -1138,7 +1218,10 @@ int tc_gsub(const Geometry &g)
 
 bool tc_supported(const Geometry &g)
 {
-    if (g.variant != DGE_VARIANT_SCORED || (g.d != 64 && g.d != 128) || g.m > 256 || g.G > 256)
+    // The observation rows must lie in the protected tail (t >= m), so that phase 2 needs no
+    // causal mask; the caller's rare t < m goes to the warp-level kernels.
+    if (g.variant != DGE_VARIANT_SCORED || (g.d != 64 && g.d != 128) || g.m > 256 || g.G > 256 ||
+        g.tail < g.m)
         return false;
     const int gs = tc_gsub(g);
     if (gs == 0 || (size_t)((gs * g.m + 3) & ~3) * 4 > (size_t)kStageBytes)
@@ -1159,36 +1242,29 @@ TcPlan tc_plan(const Geometry &g)
     p.r_pad = (p.rows + 15) & ~15;
     p.r4 = (p.rows + 3) & ~3;
     p.nslab = g.d / 64;
-    // Key chunk (one task): as long as the phase-1 data of the tasks between an item's two
-    // phases still fits in L2, i.e. (S + nchunks) chunks of K rows <= L2, which is about
-    // chunk <= (L2 / row_bytes - n) / S.  Longer tasks load the query block less often and
-    // pay the per-task hand-offs less often; measured on GB300 at 32K keys, 24 tiles
-    // (3072 keys) ran 11% faster than 8 and a 32-tile chunk lost L2 hits.  Rounded to a
-    // multiple of 8 tiles, within 8 .. 32 tiles, and at most a quarter of a unit (rounded down
-    // to 8 tiles): short units need enough items to fill the steps -- at 8K keys, 16-tile
-    // chunks (4 per unit) ran 6% faster than 24-tile ones (3 per unit, 5 steps on 152 CTAs).
-    int dev = 0, l2 = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        sms <= 0)
-        l2 = 0, sms = 1;
-    const double row_bytes = (double)g.d * 2.0;
-    double fit = ((double)l2 / row_bytes - (double)g.n) / (double)sms / kTile;
-    int tiles = (int)(fit / 8.0 + 0.5) * 8;
-    tiles = tiles < 8 ? 8 : (tiles > 32 ? 32 : tiles);
+    // Key chunk (one task).  The phase-1 data read between an item's two phases is about
+    // (lag + nchunks) chunks, so short chunks keep the phase-2 re-read in L2; longer ones pay
+    // the per-task hand-offs (the row-sum reduction, the lse staging, a query-block load) less
+    // often.  Whole units take kChunkTiles tiles (fewer when the unit is shorter); a unit is
+    // split into chunks of equal length (within a tile).
     const int unit_tiles = (g.n + kTile - 1) / kTile;
-    const int quarter = (unit_tiles / 4) / 8 * 8;
+    int tiles = kChunkTiles < unit_tiles ? kChunkTiles : unit_tiles;
     // Row blocks (R > 144) make the kernel bound by the tensor pipe and the epilogue, not by
     // DRAM, so the L2 fit does not matter and the longest chunk wins: at 128K keys and four
     // row blocks (70B shape), quarter-unit chunks (256 tiles) took 25.4 ms against 26.7 ms
     // for 16-tile ones.
+    const int quarter = (unit_tiles / 4) / 8 * 8;
     if (p.nrb > 1)
-        tiles = quarter < 8 ? 8 : quarter;
-    if (tiles > quarter)
-        tiles = quarter < 8 ? 8 : quarter;
+        tiles = quarter < 8 ? (unit_tiles < 8 ? unit_tiles : 8) : quarter;
     p.chunk_keys = tiles * kTile;
-    p.nchunks = (g.n + p.chunk_keys - 1) / p.chunk_keys;
+    p.nchunks = (unit_tiles + tiles - 1) / tiles;
+    // Chunks whose keys start below n - m carry phase-1 keys (the first p1_chunks ones).
+    const int first_obs = g.n - g.m;
+    p.p1_chunks = 0;
+    for (int c = 0; c < p.nchunks; ++c)
+        if ((int)((int64_t)c * unit_tiles / p.nchunks) * kTile < first_obs)
+            p.p1_chunks = c + 1;
+    p.nparts = p.nchunks + 1;
 
     p.kstages = kMaxKStages;
     while (p.kstages > 2 && smem_bytes(p.r_pad, p.nslab, p.kstages) > 232448)
@@ -1233,6 +1309,8 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
     a.kstages = plan.kstages;
     a.unit_tiles = (g.n + kTile - 1) / kTile;
     a.nchunks = plan.nchunks;
+    a.p1_chunks = plan.p1_chunks;
+    a.nparts = plan.nparts;
     a.lse_in = buf.lse_in;
     if (a.lse_in) {
         // One pass, nothing to keep in L2: tasks of up to 32 tiles.
@@ -1246,9 +1324,20 @@ cudaError_t launch_score_tc(const TensorDesc &K, const TensorDesc &Q, const Geom
         base += a.ng[w];
     }
     const int64_t grid = a.items < sms ? a.items : sms;
-    a.lag = a.lse_in ? 0 : a.nchunks - 1;
-    // Phase 2 of the last item runs in step `steps`: (steps - 1) * grid + s - lag covers it.
-    a.steps = (a.items + a.lag + grid - 1) / grid;
+    if (a.lse_in) {
+        a.lag = 0;
+        a.total = a.items;
+    } else {
+        // Phase 2 of an item is claimed `lag` items after its phase 1: the whole unit's
+        // chunks (nchunks - 1) plus about one and a half rounds of the grid, so that the
+        // phase-1 tasks it needs, claimed that much earlier, have finished (each CTA holds at
+        // most about two tasks between claiming and finishing them) while the chunk is still
+        // in L2.
+        const int64_t lag = (int64_t)kLagGridX10 * grid / 10 + a.nchunks - 1;
+        a.lag = lag < a.items ? lag : a.items;
+        a.total = 2 * a.items;
+    }
+    a.claim = buf.claim;
     a.part = buf.part;
     a.lse2 = buf.lse2;
     a.raw = buf.raw;
