@@ -431,135 +431,164 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
     if (warp < kEpiWarp0) {
         ptx::regs_dec<kRegsControl>();
     if (warp == 0) {
-        // ---- TMA producer ---------------------------------------------------------------
+        // ---- TMA producer (the whole warp: lane 0 claims, arms the barriers and publishes;
+        // the boxes of a copy are spread over the lanes, one box each) ----------------------
         if (lane == 0) {
             ptx::prefetch_tmap(&tmK);
             ptx::prefetch_tmap(&tmQ);
-            // Phase-1 tiles stay in L2 for the phase-2 re-read one step later; the re-read
-            // marks them first to go.
-            const uint64_t keep = ptx::make_policy_evict_last();
-            const uint64_t drop = ptx::make_policy_evict_first();
-            int ks = 0, ptc = 0;
-            uint32_t kph = 0;
-            long long cy_wq = 0, cy_wk = 0;
-            const long long cy0 = tclock<kTr>();
-            bool ok = true;
-            // Tasks are handed on one ahead: the next task is claimed kClaimAhead tiles before
-            // the current one's last copy, published to the ring one tile later, and its query
-            // block loaded as soon as that buffer is free, so neither the claim's round trip
-            // nor the query copy falls between two tasks.  Task k uses query buffer k & 1.
-            auto claim_next = [&](uint32_t first, Task &N) -> int64_t {
-                for (uint32_t c = first; (int64_t)c < a.total; c = atomicAdd(a.claim, 1u))
-                    if (task_at(a, c, N))
-                        return c;
-                return -1;
-            };
-            auto publish = [&](int k, int64_t pos) -> bool {
-                const int slot = k % kRing;
-                if (!wait_bar(&sm.bar[kBarRingEmpty + slot], (uint32_t)((k / kRing) & 1) ^ 1u,
-                              flag, a))
-                    return false;
+        }
+        // Phase-1 tiles stay in L2 for the phase-2 re-read; the re-read marks them first to go.
+        const uint64_t keep = ptx::make_policy_evict_last();
+        const uint64_t drop = ptx::make_policy_evict_first();
+        int ks = 0, ptc = 0;
+        uint32_t kph = 0;
+        long long cy_wq = 0, cy_wk = 0;
+        const long long cy0 = tclock<kTr>();
+        bool ok = true;
+        // A bounded wait with a warp-uniform outcome.
+        auto wait_w0 = [&](uint64_t *bar, uint32_t parity) -> bool {
+            const bool got = wait_bar(bar, parity, flag, a);
+            return __all_sync(0xffffffffu, got);
+        };
+        // Tasks are handed on one ahead: the next task is claimed kClaimAhead tiles before the
+        // current one's last copy (lane 0's atomic; its value is read one tile later, so the
+        // round trip is hidden), published to the ring then, and its query block loaded as
+        // soon as that buffer is free, so neither the claim nor the query copy falls between
+        // two tasks.  Task k uses query buffer k & 1.
+        auto claim_one = [&]() -> uint32_t {
+            uint32_t c = 0;
+            if (lane == 0)
+                c = atomicAdd(a.claim, 1u);
+            return __shfl_sync(0xffffffffu, c, 0);
+        };
+        auto claim_next = [&](uint32_t first, Task &N) -> int64_t {
+            for (uint32_t c = first; (int64_t)c < a.total; c = claim_one())
+                if (task_at(a, c, N))
+                    return c;
+            return -1;
+        };
+        auto publish = [&](int k, int64_t pos) -> bool {
+            const int slot = k % kRing;
+            if (!wait_w0(&sm.bar[kBarRingEmpty + slot], (uint32_t)((k / kRing) & 1) ^ 1u))
+                return false;
+            if (lane == 0) {
                 sm.ring[slot] = pos;
                 ptx::mbar_arrive(&sm.bar[kBarRingFull + slot]);
-                return true;
-            };
-            auto load_q = [&](const Task &N, int b, uint32_t ph) {
-                int l, bb, h;
-                unit_coords(g, kFx ? N.u / a.nrb : N.u, l, bb, h);
-                const int qhead = h * g.G + (kFx ? (int)(N.u % a.nrb) * a.gsub : 0);
+            }
+            return true;
+        };
+        auto load_q = [&](const Task &N, int b, uint32_t ph) {
+            int l, bb, h;
+            unit_coords(g, kFx ? N.u / a.nrb : N.u, l, bb, h);
+            const int qhead = h * g.G + (kFx ? (int)(N.u % a.nrb) * a.gsub : 0);
+            if (lane == 0) {
                 ptx::mbar_arrive_expect_tx(&sm.bar[kBarQFull + b],
                                            (uint32_t)a.nslab * 128u * (uint32_t)a.rows);
                 flag[kFlagQArm + b] = (int)ph;
-                for (int s = 0; s < a.nslab; ++s)
-                    ptx::tma_load_5d_hint(sm.q + ((size_t)b * a.nslab + s) * q_slab_bytes, &tmQ,
-                                          &sm.bar[kBarQFull + b], s * 64, 0, qhead, bb, l, keep);
-            };
-            Task T;
-            int64_t p = claim_next(atomicAdd(a.claim, 1u), T);
-            ok = publish(0, p);
-            bool q_ready = false;  // the current task's query block is already on its way
-            for (int k = 0; ok && p >= 0; ++k) {
-                const int qb = k & 1;
-                const uint32_t qph = (uint32_t)((k >> 1) & 1);
-                if (!q_ready) {
-                    long long c0 = tclock<kTr>();
-                    if (!wait_bar(&sm.bar[kBarQEmpty + qb], qph ^ 1, flag, a)) {
-                        ok = false;
-                        break;
-                    }
-                    cy_wq += tclock<kTr>() - c0;
-                    load_q(T, qb, qph);
-                }
-                int l, bb, h;
-                unit_coords(g, kFx ? T.u / a.nrb : T.u, l, bb, h);
-                Task N;
-                int64_t np = -1;
-                uint32_t pend = 0;
-                bool claimed = false, pushed = false, nq = false;
-                const int claim_at = max(T.ntiles - kClaimAhead, 0);
-                const int nqb = qb ^ 1;
-                const uint32_t nqph = (uint32_t)(((k + 1) >> 1) & 1);
-                const uint64_t pol = T.phase == 2 ? drop : keep;
-                int w0 = 0;               // first key of the page-id window (paged caches)
-                const int *ids = sm.pages;
-                for (int tile = 0; tile < T.ntiles; ++tile) {
-                    if (tile == claim_at) {
-                        pend = atomicAdd(a.claim, 1u);
-                        claimed = true;
-                    } else if (claimed && !pushed) {
-                        np = claim_next(pend, N);
-                        if (!publish(k + 1, np)) {
-                            ok = false;
-                            break;
-                        }
-                        pushed = true;
-                    }
-                    if (pushed && np >= 0 && !nq &&
-                        ptx::mbar_test_parity(&sm.bar[kBarQEmpty + nqb], nqph ^ 1)) {
-                        load_q(N, nqb, nqph);
-                        nq = true;
-                    }
-                    if constexpr (kPaged) {
-                        if (tile % tc::kPageWindowTiles == 0) {
-                            w0 = T.k_lo + tile * kTile;
-                            ids = tc::fetch_pages(sm.pages, a.kp, bb, w0,
-                                                  min(T.ntiles - tile, tc::kPageWindowTiles));
-                        }
-                    }
-                    long long c0 = tclock<kTr>();
-                    if (!wait_bar(&sm.bar[kBarKEmpty + ks], kph ^ 1, flag, a)) {
-                        ok = false;
-                        break;
-                    }
-                    cy_wk += tclock<kTr>() - c0;
-                    trace_at<kTr>(a, kTrTileIssue, ptc++);
-                    ptx::mbar_arrive_expect_tx(&sm.bar[kBarKFull + ks],
-                                               (uint32_t)a.nslab * kSlabBytes);
-                    flag[kFlagKArm + ks] = (int)kph;
-                    tc::load_k_tile<kPaged>(sm.k + (size_t)ks * a.nslab * kSlabBytes,
-                                            kSlabBytes, a.nslab, &tmK, &tmKm,
-                                            &sm.bar[kBarKFull + ks], T.k_lo + tile * kTile, l,
-                                            bb, h, a.kp, ids, w0, pol);
-                    if (++ks == a.kstages) {
-                        ks = 0;
-                        kph ^= 1;
-                    }
-                }
-                if (!ok)
+            }
+            __syncwarp();
+            if (lane < a.nslab)
+                ptx::tma_load_5d_hint(sm.q + ((size_t)b * a.nslab + lane) * q_slab_bytes, &tmQ,
+                                      &sm.bar[kBarQFull + b], lane * 64, 0, qhead, bb, l, keep);
+        };
+        Task T;
+        int64_t p = claim_next(claim_one(), T);
+        ok = publish(0, p);
+        bool q_ready = false;  // the current task's query block is already on its way
+        for (int k = 0; ok && p >= 0; ++k) {
+            const int qb = k & 1;
+            const uint32_t qph = (uint32_t)((k >> 1) & 1);
+            if (!q_ready) {
+                long long c0 = tclock<kTr>();
+                if (!wait_w0(&sm.bar[kBarQEmpty + qb], qph ^ 1)) {
+                    ok = false;
                     break;
-                if (!claimed)
-                    pend = atomicAdd(a.claim, 1u);
-                if (!pushed) {
-                    np = claim_next(pend, N);
+                }
+                cy_wq += tclock<kTr>() - c0;
+                load_q(T, qb, qph);
+            }
+            int l, bb, h;
+            unit_coords(g, kFx ? T.u / a.nrb : T.u, l, bb, h);
+            Task N;
+            int64_t np = -1;
+            uint32_t pend = 0;  // lane 0's claimed position (valid once read after a tile)
+            bool claimed = false, pushed = false, nq = false;
+            const int claim_at = max(T.ntiles - kClaimAhead, 0);
+            const int nqb = qb ^ 1;
+            const uint32_t nqph = (uint32_t)(((k + 1) >> 1) & 1);
+            const uint64_t pol = T.phase == 2 ? drop : keep;
+            int w0 = 0;               // first key of the page-id window (paged caches)
+            const int *ids = sm.pages;
+            for (int tile = 0; tile < T.ntiles; ++tile) {
+                if (tile == claim_at) {
+                    if (lane == 0)
+                        pend = atomicAdd(a.claim, 1u);
+                    claimed = true;
+                } else if (claimed && !pushed) {
+                    np = claim_next(__shfl_sync(0xffffffffu, pend, 0), N);
                     if (!publish(k + 1, np)) {
                         ok = false;
                         break;
                     }
+                    pushed = true;
                 }
-                T = N;
-                p = np;
-                q_ready = nq;
+                if (pushed && np >= 0 && !nq &&
+                    __shfl_sync(0xffffffffu,
+                                ptx::mbar_test_parity(&sm.bar[kBarQEmpty + nqb], nqph ^ 1) ? 1
+                                                                                            : 0,
+                                0)) {
+                    load_q(N, nqb, nqph);
+                    nq = true;
+                }
+                if constexpr (kPaged) {
+                    if (tile % tc::kPageWindowTiles == 0) {
+                        w0 = T.k_lo + tile * kTile;
+                        if (lane == 0)
+                            tc::fetch_pages(sm.pages, a.kp, bb, w0,
+                                            min(T.ntiles - tile, tc::kPageWindowTiles));
+                        __syncwarp();
+                        ids = tc::page_ids_at(sm.pages, a.kp, bb, w0);
+                    }
+                }
+                long long c0 = tclock<kTr>();
+                if (!wait_w0(&sm.bar[kBarKEmpty + ks], kph ^ 1)) {
+                    ok = false;
+                    break;
+                }
+                cy_wk += tclock<kTr>() - c0;
+                if (lane == 0) {
+                    trace_at<kTr>(a, kTrTileIssue, ptc);
+                    ptx::mbar_arrive_expect_tx(&sm.bar[kBarKFull + ks],
+                                               (uint32_t)a.nslab * kSlabBytes);
+                    flag[kFlagKArm + ks] = (int)kph;
+                }
+                ++ptc;
+                __syncwarp();
+                tc::load_k_tile_warp<kPaged>(sm.k + (size_t)ks * a.nslab * kSlabBytes,
+                                             kSlabBytes, a.nslab, &tmK, &tmKm,
+                                             &sm.bar[kBarKFull + ks], T.k_lo + tile * kTile, l,
+                                             bb, h, a.kp, ids, w0, pol, lane);
+                if (++ks == a.kstages) {
+                    ks = 0;
+                    kph ^= 1;
+                }
             }
+            if (!ok)
+                break;
+            if (!claimed && lane == 0)
+                pend = atomicAdd(a.claim, 1u);
+            if (!pushed) {
+                np = claim_next(__shfl_sync(0xffffffffu, pend, 0), N);
+                if (!publish(k + 1, np)) {
+                    ok = false;
+                    break;
+                }
+            }
+            T = N;
+            p = np;
+            q_ready = nq;
+        }
+        if (lane == 0) {
             trace_put<kTr>(a, kTrProdWaitQ, cy_wq);
             trace_put<kTr>(a, kTrProdWaitK, cy_wk);
             trace_put<kTr>(a, kTrProdTotal, tclock<kTr>() - cy0);

@@ -140,6 +140,13 @@ __device__ __forceinline__ const int *fetch_pages_issue(int *buf, const KPaging 
     return ids;
 }
 
+// Where fetch_pages(buf, pg, bb, k0, ...) puts the page ids (any thread can compute it).
+__device__ __forceinline__ const int *page_ids_at(int *buf, const KPaging &pg, int bb, int k0)
+{
+    const int32_t *src = pg.bt + (int64_t)bb * pg.pps + k0 / pg.page_size;
+    return buf + (int)(((uintptr_t)src >> 2) & 3);
+}
+
 // Waits for every page-id copy this thread has issued.
 __device__ __forceinline__ void fetch_pages_wait()
 {
@@ -208,6 +215,61 @@ __device__ __forceinline__ void load_k_tile(uint8_t *dst, uint32_t slab_bytes, i
             for (int s = 0; s < nslab; ++s)
                 ptx::tma_load_5d_hint(dst + s * slab_bytes + (j << pg.ps_shift) * 128, map, bar,
                                       s * 64, h, 0, page, l, policy);
+        }
+    }
+}
+
+// load_k_tile issued by a whole warp, one box per lane: box i of a tile is slab i % nslab of
+// page i / nslab (nslab boxes for a contiguous cache, a page of 128 slots or more, or a run
+// of consecutive pages).  The caller arms `bar` for the whole tile before any lane issues.
+template <bool kPaged>
+__device__ __forceinline__ void load_k_tile_warp(uint8_t *dst, uint32_t slab_bytes, int nslab,
+                                                 const CUtensorMap *map,
+                                                 const CUtensorMap *merged, uint64_t *bar,
+                                                 int k0, int l, int bb, int h, const KPaging &pg,
+                                                 const int *ids, int w0, uint64_t policy,
+                                                 int lane)
+{
+    if constexpr (!kPaged) {
+        if (lane < nslab)
+            ptx::tma_load_5d_hint(dst + lane * slab_bytes, map, bar, lane * 64, k0, h, bb, l,
+                                  policy);
+    } else if (pg.page_size >= 128) {
+        int page = 0, slot = 0;
+        if (k0 < pg.n) {
+            const int pi = k0 / pg.page_size;
+            const int pid = ids[pi - w0 / pg.page_size];
+            page = (unsigned)pid < (unsigned)pg.num_pages ? pid : 0;
+            slot = k0 - pi * pg.page_size;
+        }
+        if (lane < nslab)
+            ptx::tma_load_5d_hint(dst + lane * slab_bytes, map, bar, lane * 64, h, slot, page, l,
+                                  policy);
+    } else {
+        const int npg = 128 >> pg.ps_shift;
+        const int i0 = (k0 - w0) >> pg.ps_shift;
+        const int valid = (pg.n - k0 + pg.page_size - 1) >> pg.ps_shift;
+        if (pg.merged && valid >= npg) {
+            const int first = ids[i0];
+            bool run = (unsigned)first <= (unsigned)(pg.num_pages - npg);
+            for (int j = 1; j < npg; ++j)
+                run = run && ids[i0 + j] == first + j;
+            if (run) {
+                if (lane < nslab)
+                    ptx::tma_load_5d_hint(dst + lane * slab_bytes, merged, bar, lane * 64, h,
+                                          first << pg.ps_shift, l, 0, policy);
+                return;
+            }
+        }
+        const int j = lane / nslab, s = lane - j * nslab;
+        if (j < npg) {
+            int page = 0;
+            if (j < valid) {
+                const int pid = ids[i0 + j];
+                page = (unsigned)pid < (unsigned)pg.num_pages ? pid : 0;
+            }
+            ptx::tma_load_5d_hint(dst + s * slab_bytes + (j << pg.ps_shift) * 128, map, bar,
+                                  s * 64, h, 0, page, l, policy);
         }
     }
 }
