@@ -27,6 +27,8 @@
 #include <math.h>
 #include <string.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "kernels.h"
 #include "tc_common.cuh"
@@ -200,10 +202,13 @@ __device__ __forceinline__ uint32_t causal_mask(int key, int p0, int pb, int cb)
 }
 
 // Phase 1 for one 16-column group: z[c] += 2^{x_c} (keys after a row's position add nothing).
-__device__ __forceinline__ void rows_add(float (&z)[16], const float (&v)[16], float s2, bool diag,
-                                         int key, int p0, int pb, int cb)
+// kDiag: the tile reaches the block's own positions (masked); a compile-time choice, so the
+// loop over the other tiles carries no mask code.
+template <bool kDiag>
+__device__ __forceinline__ void rows_add(float (&z)[16], const float (&v)[16], float s2, int key,
+                                         int p0, int pb, int cb)
 {
-    if (!diag) {
+    if constexpr (!kDiag) {
         const float2 sc = make_float2(s2, s2);
 #pragma unroll
         for (int c = 0; c < 16; c += 2) {
@@ -227,11 +232,12 @@ __device__ __forceinline__ void rows_add(float (&z)[16], const float (&v)[16], f
 // holds -lse (rows past the cache or padding: -inf).  Columns 2q, 2q+1 go to acc[q % 4]: four
 // independent chains of additions instead of one (the epilogue is latency-bound), added
 // together in a fixed order at the end of the task.
+template <bool kDiag>
 __device__ __forceinline__ void col_add(float2 (&acc)[4], const float (&v)[16],
-                                        const float (&nL)[16], float s2, bool diag, int key,
-                                        int p0, int pb, int cb)
+                                        const float (&nL)[16], float s2, int key, int p0, int pb,
+                                        int cb)
 {
-    if (!diag) {
+    if constexpr (!kDiag) {
         const float2 sc = make_float2(s2, s2);
 #pragma unroll
         for (int c = 0; c < 16; c += 2) {
@@ -643,12 +649,13 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
 #pragma unroll
                     for (int c = 0; c < 16; ++c)
                         z[i][c] = 0.f;
-                for (int i = 0; i < T.ntiles; ++i, ++tc) {
+                // Tiles below the block's first position are seen by every row (no mask); the
+                // rest reach the block's own positions.  Two loops, each with its own body.
+                auto tile1 = [&](int i, auto diag_c) {
+                    constexpr bool kDiag = decltype(diag_c)::value;
                     const int ab = tc % kAccBufs;
                     const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
-                    const int k0 = i * kTile;
-                    const int key = k0 + kl;
-                    const bool diag = k0 + kTile > p0;  // the tile reaches the block's rows
+                    const int key = i * kTile + kl;
                     if (acquire_acc(ab, aph)) {
                         const uint32_t tbase =
                             tmem_base + (uint32_t)(ab * a.acc_stride + col_base) + lane_off;
@@ -656,11 +663,18 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
 #pragma unroll
                             for (int gj = 0; gj < kMaxGroups; ++gj)
                                 if (gj == gi)
-                                    rows_add(z[gj], v, s2, diag, key, p0, a.pb, col_base + gj * 16);
+                                    rows_add<kDiag>(z[gj], v, s2, key, p0, a.pb,
+                                                    col_base + gj * 16);
                         });
                     }
                     release_acc(ab);
-                }
+                    ++tc;
+                };
+                const int nplain = min(T.ntiles, p0 / kTile);
+                for (int i = 0; i < nplain; ++i)
+                    tile1(i, std::false_type());
+                for (int i = nplain; i < T.ntiles; ++i)
+                    tile1(i, std::true_type());
                 // Sums over this warp's 32 keys, handed to warp 3 through a double-buffered
                 // area (it adds the lane quarters in a fixed order).
 #pragma unroll
@@ -705,11 +719,13 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
                     acc[q] = make_float2(0.f, 0.f);
-                for (int i = 0; i < T.ntiles; ++i, ++tc) {
+                // The first blocks hold rows before some of the tile's keys (masked); the rest see
+                // every key.  Two loops, each with its own body.
+                auto tile2 = [&](int i, auto diag_c) {
+                    constexpr bool kDiag = decltype(diag_c)::value;
                     const int ab = tc % kAccBufs;
                     const uint32_t aph = (uint32_t)((tc / kAccBufs) & 1);
                     const int p0 = (T.first + i) * a.pb;
-                    const bool diag = p0 < k0 + kTile;  // some row precedes some key
                     const int sub = (int)(nb % kLseGroup);
                     const int slot = (int)((nb / kLseGroup) % kLseSlots);
                     if (sub == 0)
@@ -739,7 +755,7 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                                     nl[4 * q + 3] = f.w;
                                 }
                                 ptx::tmem_ld_wait_dep(v);
-                                col_add(acc, v, nl, s2, diag, key, p0, a.pb, col_base + gi * 16);
+                                col_add<kDiag>(acc, v, nl, s2, key, p0, a.pb, col_base + gi * 16);
                             }
                     }
                     // Every warp has read this block's -lse: the fourth block of a group frees
@@ -750,7 +766,15 @@ h2o_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ C
                             ptx::mbar_arrive(&sm.bar[kBarLseEmpty + slot]);
                     }
                     release_acc(ab);
-                }
+                    ++tc;
+                };
+                // Block i is masked while its first position precedes the tile's last key.
+                const int ndiag =
+                    min(T.ntiles, max(0, (k0 + kTile + a.pb - 1) / a.pb - T.first));
+                for (int i = 0; i < ndiag; ++i)
+                    tile2(i, std::true_type());
+                for (int i = ndiag; i < T.ntiles; ++i)
+                    tile2(i, std::false_type());
                 // The three warps of this lane quarter (one per warpgroup) leave their sums in
                 // shared memory; a warp whose arrival completes the phase adds them in
                 // warpgroup order and stores the key's score (two may both see it complete:
