@@ -34,7 +34,6 @@
 #include <math.h>
 #include <string.h>
 
-#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -50,10 +49,11 @@ constexpr int kEpiWG = 3;                 // epilogue warpgroups
 constexpr int kEpiWarps = 4 * kEpiWG;
 constexpr int kEpiWarp0 = 4;              // epilogue warps are 4 .. 15 (aligned warpgroups)
 constexpr int kThreads = (kEpiWarp0 + kEpiWarps) * 32;
-// Registers per thread after reallocation: warpgroup 0 (producer, MMA, two idle warps)
-// gives up registers to the epilogue warpgroups.  The block launches with 512 threads x 128
-// registers; 4*32*56 + 12*32*152 is exactly that.
-constexpr int kRegsLaunch = 128, kRegsControl = 56, kRegsEpilogue = 152;
+// Registers per thread after reallocation: warpgroup 0 (producer, MMA, coordinators) gives
+// up registers to the epilogue warpgroups.  The block launches with 512 threads x 128
+// registers; 4*32*64 + 12*32*144 fits in that.  (56 / 152 left the producer spilling:
+// c3 1 % and 16-slot pages 5 % slower.)
+constexpr int kRegsLaunch = 128, kRegsControl = 64, kRegsEpilogue = 144;
 static_assert(4 * 32 * kRegsControl + kEpiWarps * 32 * kRegsEpilogue <= kThreads * kRegsLaunch,
               "register split");
 constexpr int kMaxGroups = 3;             // 16-column groups per epilogue warpgroup
@@ -277,61 +277,35 @@ using tc::transpose_sum32;
 
 
 // Phase 1 for one 16-column group: z[c] += 2^{x_c} (every row sees every key of phase 1).
-// A group with exactly 8 query rows (cvalid == 8, the last group of 136 stacked rows) skips
-// the exponentials of its 8 padding columns; any other group computes all 16.
-__device__ __forceinline__ void rows_add(float (&z)[16], const float (&w)[16], float s2, bool valid,
-                                         int cvalid)
+// Padding columns (no query row) are computed too: skipping them measured slower (one more
+// branch in the loop) than their exponentials cost.
+__device__ __forceinline__ void rows_add(float (&z)[16], const float (&w)[16], float s2, bool valid)
 {
     if (!valid)
         return;
     const float2 sc = make_float2(s2, s2);
-    // Fully unrolled either way (a per-pair bound check would serialise the exponentials).
-    auto pairs = [&](auto npairs) {
 #pragma unroll
-        for (int c = 0; c < 2 * decltype(npairs)::value; c += 2) {
-            const float2 x = __fmul2_rn(make_float2(w[c], w[c + 1]), sc);
-            const float2 acc = __fadd2_rn(make_float2(z[c], z[c + 1]),
-                                          make_float2(ex2(x.x), ex2(x.y)));
-            z[c] = acc.x;
-            z[c + 1] = acc.y;
-        }
-    };
-    if (cvalid == 8)
-        pairs(std::integral_constant<int, 4>());
-    else
-        pairs(std::integral_constant<int, 8>());
+    for (int c = 0; c < 16; c += 2) {
+        const float2 x = __fmul2_rn(make_float2(w[c], w[c + 1]), sc);
+        const float2 acc = __fadd2_rn(make_float2(z[c], z[c + 1]),
+                                      make_float2(ex2(x.x), ex2(x.y)));
+        z[c] = acc.x;
+        z[c + 1] = acc.y;
+    }
 }
 
 // Phase 2 for one 16-column group: adds 2^{x_c - lse_c} over the group's rows into the
-// pair accumulator.  nL holds -lse (padded columns: -inf, so they add exactly 0; a group of
-// exactly 8 rows, cvalid == 8, skips its 8 padding columns).
-__device__ __forceinline__ void col_add(float2 &acc, const float (&w)[16], const float *nLs,
-                                        float s2, int cvalid)
+// pair accumulator.  nL holds -lse (padded columns: -inf, so they add exactly 0).
+__device__ __forceinline__ void col_add(float2 &acc, const float (&w)[16], const float (&nL)[16],
+                                        float s2)
 {
-    // -lse of the group's 16 rows, from the task's staging buffer (the same 16 values for
-    // every lane: broadcast loads).
-    float nL[16];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const float4 q = reinterpret_cast<const float4 *>(nLs)[i];
-        nL[4 * i] = q.x;
-        nL[4 * i + 1] = q.y;
-        nL[4 * i + 2] = q.z;
-        nL[4 * i + 3] = q.w;
-    }
     const float2 sc = make_float2(s2, s2);
-    auto pairs = [&](auto npairs) {
 #pragma unroll
-        for (int c = 0; c < 2 * decltype(npairs)::value; c += 2) {
-            const float2 x = __ffma2_rn(make_float2(w[c], w[c + 1]), sc,
-                                        make_float2(nL[c], nL[c + 1]));
-            acc = __fadd2_rn(acc, make_float2(ex2(x.x), ex2(x.y)));
-        }
-    };
-    if (cvalid == 8)
-        pairs(std::integral_constant<int, 4>());
-    else
-        pairs(std::integral_constant<int, 8>());
+    for (int c = 0; c < 16; c += 2) {
+        const float2 x = __ffma2_rn(make_float2(w[c], w[c + 1]), sc,
+                                    make_float2(nL[c], nL[c + 1]));
+        acc = __fadd2_rn(acc, make_float2(ex2(x.x), ex2(x.y)));
+    }
 }
 
 // Runs f(gi, v) over this warp's lane quarter of 16-column groups gi = 0 .. ng-1 (ng <=
@@ -964,8 +938,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
 #pragma unroll
                                 for (int gj = 0; gj < kMaxGroups; ++gj)
                                     if (gj == gi)
-                                        rows_add(z[gj], v, s2, valid,
-                                                 a.rows - (col_base + gj * 16));
+                                        rows_add(z[gj], v, s2, valid);
                             };
                             for_groups(tbase, ng, f1);
                             cy_math += tclock<kTr>() - c0;
@@ -1019,14 +992,37 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     ++p2c;
                     if (ew == 0 && lane == 0)
                         trace_at<kTr>(a, kTrTimeline, 2048 + 2 * (p2c - 1));
-                    // -lse of this warpgroup's columns stays in the staging buffer for the
-                    // whole task (read per group with broadcast loads); the buffer is freed
-                    // after the task's last tile.
-                    const float *nLs = sm.sL + lb * 256 + col_base;
+                    // -lse of this warpgroup's columns into registers for the whole task; the
+                    // staging buffer is then free for the coordinator's next-but-one task.
+                    // (Reading it from shared memory per group instead measured 1 % slower.)
+                    float nL[kMaxGroups][16];
                     bool task_ok = false;
-                    const bool have_lse = wait_uniform(&sm.bar[kBarLseFull + lb], lph);
-                    if (have_lse)
+                    if (wait_uniform(&sm.bar[kBarLseFull + lb], lph)) {
+                        const float4 *L4 =
+                            reinterpret_cast<const float4 *>(sm.sL + lb * 256 + col_base);
+#pragma unroll
+                        for (int gi = 0; gi < kMaxGroups; ++gi)
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float4 q = gi < ng ? L4[gi * 4 + i]
+                                                         : make_float4(-INFINITY, -INFINITY,
+                                                                       -INFINITY, -INFINITY);
+                                nL[gi][4 * i] = q.x;
+                                nL[gi][4 * i + 1] = q.y;
+                                nL[gi][4 * i + 2] = q.z;
+                                nL[gi][4 * i + 3] = q.w;
+                            }
                         task_ok = sm.sLbad[lb] == 0;
+                        __syncwarp();
+                        if (lane == 0)
+                            ptx::mbar_arrive(&sm.bar[kBarLseEmpty + lb]);
+                    } else {
+#pragma unroll
+                        for (int gi = 0; gi < kMaxGroups; ++gi)
+#pragma unroll
+                            for (int c = 0; c < 16; ++c)
+                                nL[gi][c] = -INFINITY;
+                    }
                     if (ew == 0 && lane == 0)
                         trace_at<kTr>(a, kTrTimeline, 2048 + 2 * (p2c - 1) + 1);
                     task_ok = task_ok && !dead;
@@ -1050,8 +1046,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
 #pragma unroll
                                 for (int gj = 0; gj < kMaxGroups; ++gj)
                                     if (gj == gi)
-                                        col_add(acc, v, nLs + gj * 16, s2,
-                                                a.rows - (col_base + gj * 16));
+                                        col_add(acc, v, nL[gj], s2);
                             };
                             for_groups(tbase, ng, f2);
                             cy_math2 += tclock<kTr>() - c0;
@@ -1099,10 +1094,6 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         cy_xch += tclock<kTr>() - cx;
                         release_acc(ab, 1u);
                     }
-                    // The -lse buffer is free for the coordinator's next-but-one task.
-                    __syncwarp();
-                    if (have_lse && lane == 0)
-                        ptx::mbar_arrive(&sm.bar[kBarLseEmpty + lb]);
                 }
             }
         if (ew == 0 && lane == 0) {
