@@ -75,7 +75,7 @@ constexpr int kRing = 8;                  // claimed tasks handed from the produ
 #define DGE_TC_LAG_GRID_X10 15
 #endif
 #ifndef DGE_TC_CHUNK_TILES
-#define DGE_TC_CHUNK_TILES 48
+#define DGE_TC_CHUNK_TILES 128
 #endif
 constexpr int kLagGridX10 = DGE_TC_LAG_GRID_X10;
 // The producer claims the next task this many tiles before the current task's last copy.
@@ -84,6 +84,8 @@ constexpr int kLagGridX10 = DGE_TC_LAG_GRID_X10;
 #endif
 constexpr int kClaimAhead = DGE_TC_CLAIM_AHEAD;
 constexpr int kChunkTiles = DGE_TC_CHUNK_TILES;
+// Fewest items (unit, chunk) of a launch of whole units: about three per SM of a 152-SM GB300.
+constexpr int kMinItems = 456;
 // Arrivals that free a ring slot: the MMA warp, the two coordinator warps, the epilogue warps.
 constexpr int kRingConsumers = 3 + 12;
 constexpr int kStageBytes = 12288;        // chunk sums of a unit, staged for the lse merge
@@ -1309,12 +1311,20 @@ TcPlan tc_plan(const Geometry &g)
     p.r4 = (p.rows + 3) & ~3;
     p.nslab = g.d / 64;
     // Key chunk (one task).  The phase-1 data read between an item's two phases is about
-    // (lag + nchunks) chunks, so short chunks keep the phase-2 re-read in L2; longer ones pay
-    // the per-task hand-offs (the row-sum reduction, the lse staging, a query-block load) less
-    // often.  Whole units take kChunkTiles tiles (fewer when the unit is shorter); a unit is
-    // split into chunks of equal length (within a tile).
+    // (lag + nchunks) chunks, so only chunks of about 8 tiles keep the phase-2 re-read in L2,
+    // and those pay the per-task hand-offs (the row-sum reduction, the lse staging, a
+    // query-block load) too often: at 32K keys, 8 tiles 3.09 ms, 16 tiles 2.71, 48 tiles 2.56,
+    // 128 tiles 2.51 (K read twice at the copy rate).  Whole units take chunks of at most
+    // kChunkTiles tiles, but at least kMinItems items in all when the units are few and short
+    // (8K keys, 256 units: two chunks of 32 tiles, 0.189 ms against 0.203 for whole units),
+    // never below 16 tiles; a unit is split into chunks of equal length (within a tile).
     const int unit_tiles = (g.n + kTile - 1) / kTile;
-    int tiles = kChunkTiles < unit_tiles ? kChunkTiles : unit_tiles;
+    int nch = (unit_tiles + kChunkTiles - 1) / kChunkTiles;
+    const int64_t want = (kMinItems + g.U - 1) / (g.U > 0 ? g.U : 1);
+    const int cap = unit_tiles / 16 > 1 ? unit_tiles / 16 : 1;
+    if (want > nch)
+        nch = want < cap ? (int)want : (cap > nch ? cap : nch);
+    int tiles = nch > 0 && unit_tiles > 0 ? (unit_tiles + nch - 1) / nch : 1;
     // Row blocks (R > 144) make the kernel bound by the tensor pipe and the epilogue, not by
     // DRAM, so the L2 fit does not matter and the longest chunk wins: at 128K keys and four
     // row blocks (70B shape), quarter-unit chunks (256 tiles) took 25.4 ms against 26.7 ms
