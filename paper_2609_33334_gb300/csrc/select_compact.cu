@@ -69,6 +69,7 @@ constexpr int kSmemKeys = 53248;  // candidates held in shared memory (208 KiB)
 struct SelectParams {
     Geometry g;
     LayerTable layers;
+    int64_t lead = 0;   // pool_select: a CTA prefetches the raw scores of unit u + lead into L2
 };
 
 __device__ __forceinline__ int64_t unit_row_base(const SelectParams &p, int64_t u, int &budget)
@@ -104,6 +105,7 @@ static_assert(kRadixBins == 2 * kSelThreads, "two bins per thread in the bin sea
 // Shared-memory scratch of the selection helpers.
 struct SelScratch {
     uint32_t hist[kRadixBins];
+    uint32_t bincnt;   // keys in the bin a pass selected
     int warp_a[kSelWarps], warp_b[kSelWarps], warp_c[kSelWarps];
     uint32_t prefix;
     int rank;
@@ -114,7 +116,11 @@ struct SelScratch {
 // highest bit in which the smallest and the largest key differ (the bits above are common to
 // every key), kRadixBits a pass: the scores of one unit share a few exponents, so histograms
 // of the top bits would put nearly every key in a handful of bins, whose shared-memory atomics
-// serialise.  Called by every thread of a block of kSelThreads.
+// serialise.  The passes stop early when every key of the selected bin is kept (its count is
+// the rank still wanted): T is then the bin's lowest possible key (the prefix, lower bits
+// zero) and need_eq = C, which keeps exactly the keys >= T.  After two 11-bit passes the bin
+// nearly always holds one key, so the third pass is skipped.  Called by every thread of a
+// block of kSelThreads.
 template <typename KeyAt>
 __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, uint32_t &T,
                                 int &need_eq, uint32_t kmin = 0xffffffffu, uint32_t kmax = 0u,
@@ -151,6 +157,7 @@ __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, u
     uint32_t prefix = kmax & mask;
     int rank = keep;  // 1-based rank of T among the keys matching `prefix`, from the top
     const int npass = (top + kRadixBits) / kRadixBits;
+    bool whole_bin = false;
 #pragma unroll 1
     for (int pass = 0; pass < npass; ++pass) {
         const int hi = top - kRadixBits * pass;         // highest bit of this pass
@@ -198,15 +205,20 @@ __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, u
                 const bool hi_bin = run + c_hi >= (uint32_t)rank;
                 sc.prefix = prefix | ((uint32_t)(hi_bin ? tb : tb - 1) << shift);
                 sc.rank = rank - (int)(hi_bin ? run : run + c_hi);
+                sc.bincnt = hi_bin ? c_hi : c_lo;
             }
         }
         __syncthreads();
         prefix = sc.prefix;
         rank = sc.rank;
         mask |= bmask << shift;
+        if ((uint32_t)rank == sc.bincnt) {   // the whole bin is kept
+            whole_bin = true;
+            break;
+        }
     }
     T = npass == 0 ? kmax : prefix;   // npass == 0: every key is equal
-    need_eq = rank;
+    need_eq = whole_bin ? C : rank;
 }
 
 // Writes the positions s0 + j of the kept keys -- every key above T and the first need_eq keys
@@ -457,6 +469,18 @@ pool_select_kernel(const float *__restrict__ raw, float *__restrict__ pooled_out
 
     // Raw scores to shared memory, pooled values to registers, then keys in place.
     const float *row = raw + u * (int64_t)P;
+    // The unit that will most likely take this SM next (one CTA per SM: u + the SM count) has
+    // its raw scores prefetched into L2 now, so its load comes from L2.  Only whole 16-byte
+    // pieces inside that row are named (the bulk prefetch's alignment rule).
+    if (tid == 0 && p.lead > 0 && u + p.lead < g.U) {
+        const uintptr_t a0 = reinterpret_cast<uintptr_t>(raw + (u + p.lead) * (int64_t)P);
+        const uintptr_t lo = (a0 + 15) & ~uintptr_t(15);
+        const uintptr_t hi = (a0 + (uintptr_t)P * 4) & ~uintptr_t(15);
+        if (hi > lo)
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(lo),
+                         "r"((uint32_t)(hi - lo))
+                         : "memory");
+    }
     uint32_t *skey = sbuf + kPsGuard;
     float *sraw = reinterpret_cast<float *>(skey);
     for (int j = tid; j < P; j += kPsThreads)
@@ -580,6 +604,13 @@ cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, cons
     SelectParams p;
     p.g = g;
     p.layers = layers;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess)
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess)
+        return e;
+    p.lead = sms;
     // The row rounded up to whole 128-position chunks, with guard cells on both sides.
     const size_t smem = (size_t)(((max(g.P, 1) + 127) & ~127) + 2 * kPsGuard) * sizeof(uint32_t);
     using KernT = void (*)(const float *, float *, int32_t *, SelectParams, int);
