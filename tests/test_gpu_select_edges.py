@@ -99,3 +99,28 @@ def test_fused_select_crafted(kind):
     for u in range(p.U):
         np.testing.assert_array_equal(idx[u * B:(u + 1) * B],
                                       expected(scores[u], wl.n, wl.sinks, wl.tail, B))
+
+
+@pytest.mark.parametrize("n", [3000, 40000, 70000])
+@pytest.mark.parametrize("extra", [0, 1, -1])
+def test_select_whole_bin(n, extra):
+    """keep + extra large candidates (1000 plus less than 0.5, so they share exponent and top
+    mantissa bits) among small ones.  With extra = 0 the first radix pass selects a bin that
+    is kept whole, several distinct keys in it, and the passes stop there with the bin's
+    lowest possible key as the threshold; with extra = +1 the threshold falls inside that bin,
+    with extra = -1 among the small keys."""
+    wl = inputs.WORKLOADS["c1_tiny"].with_(L=1, b=1, Hq=4, Hkv=2, n=n, budgets=(n // 7,),
+                                           sinks=4)
+    p = api.problem_from_workload(wl)
+    B = wl.budgets[0]
+    keep = B - wl.sinks - wl.tail
+    rng = np.random.default_rng(n * 10 + extra + 1)
+    base = rng.uniform(1e-4, 2e-4, (p.U, p.P)).astype(np.float32)
+    for u in range(p.U):
+        pos = rng.choice(np.arange(wl.sinks, p.P), keep + extra, replace=False)
+        base[u, pos] = (1000.0 + 0.5 * rng.random(keep + extra)).astype(np.float32)
+    idx = api.select(p, torch.from_numpy(base).cuda()).cpu().numpy()
+    for u in range(p.U):
+        np.testing.assert_array_equal(idx[u * B:(u + 1) * B],
+                                      expected(base[u], n, wl.sinks, wl.tail, B),
+                                      err_msg=f"extra {extra}")
