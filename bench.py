@@ -185,14 +185,26 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS_SUSTAINED, "fallback"
 
 
-def source_digest():
-    """sha256 over the kernel sources (ties an ncu traffic figure to the code it measured)."""
+# The source file of each kernel whose DRAM traffic profiles/dram_traffic.txt records.
+KERNEL_SOURCE = {"score_tc": "score_tc.cu", "h2o_tc_lse": "h2o_tc.cu",
+                 "h2o_tc_colsum": "h2o_tc.cu", "pool_select": "select_compact.cu",
+                 "compact": "select_compact.cu", "select": "select_compact.cu"}
+
+
+def source_digest(kernel=None):
+    """sha256 over a kernel's source file and every shared header (csrc/*.cuh, csrc/*.h,
+    include/dge.h), or over all kernel sources when `kernel` is None or unknown.  It ties an
+    ncu traffic figure to the code it measured: a change to another kernel's file leaves the
+    figure valid, a change to this kernel or to a header voids it."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_33334_gb300", "csrc")
-    for fn in sorted(os.listdir(csrc)):
-        if fn.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, fn), "rb") as f:
-                h.update(fn.encode() + f.read())
+    own = KERNEL_SOURCE.get(kernel)
+    files = [os.path.join(csrc, fn) for fn in sorted(os.listdir(csrc))
+             if fn.endswith((".cuh", ".h")) or (fn.endswith(".cu") and (own is None or fn == own))]
+    files.append(os.path.join(ROOT, "include", "dge.h"))
+    for path in files:
+        with open(path, "rb") as f:
+            h.update(os.path.basename(path).encode() + f.read())
     return h.hexdigest()[:16]
 
 
@@ -201,7 +213,7 @@ def ncu_traffic(kernel, workload):
     path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
     if not os.path.exists(path):
         return None
-    digest = source_digest()
+    digest = source_digest(kernel)
     with open(path) as f:
         for line in f:
             parts = line.split()
