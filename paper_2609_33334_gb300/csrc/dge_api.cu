@@ -699,9 +699,14 @@ int evict_impl(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t w
     float *raw = ws_at<float>(ws, plan.off_raw);
     const float *sel = raw;
     const bool fused = g.select_block < 2 && pool_select_supported(g);
+    const bool fused_large = !fused && g.select_block < 2 && pool_select_large_supported(g);
     if (fused) {
         DGE_LAUNCH("pool_select", stream,
                    launch_pool_select(g, plan.layers, raw, bufs->scores, bufs->idx, stream));
+    } else if (fused_large) {
+        float *pooled = bufs->scores ? bufs->scores : ws_at<float>(ws, plan.off_pooled);
+        DGE_LAUNCH("pool_select", stream,
+                   launch_pool_select_large(g, plan.layers, raw, pooled, bufs->idx, stream));
     } else if (g.pool != DGE_POOL_NONE) {
         float *pooled = bufs->scores ? bufs->scores : ws_at<float>(ws, plan.off_pooled);
         DGE_LAUNCH("pool", stream,
@@ -715,7 +720,7 @@ int evict_impl(const dge_problem *p, const dge_buffers *bufs, void *ws, size_t w
     if (g.select_block >= 2)
         DGE_LAUNCH("block_select", stream,
                    launch_block_select(g, plan.layers, sel, bufs->idx, stream));
-    else if (!fused)
+    else if (!fused && !fused_large)
         DGE_LAUNCH("select", stream, launch_select(g, plan.layers, sel, bufs->idx, stream));
     if (inplace)
         DGE_LAUNCH("compact_inplace", stream,

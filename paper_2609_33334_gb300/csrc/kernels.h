@@ -134,6 +134,11 @@ cudaError_t launch_heldout(const TensorDesc &Qh, const TensorDesc &K, const Tens
 bool pool_select_supported(const Geometry &g);
 cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, const float *raw,
                                float *pooled_out, int32_t *idx, cudaStream_t stream);
+// The same for longer rows (P > 32768; avg or max pooling of radius <= 4): the pooled scores
+// go to `pooled` (required: the selection reads them back).
+bool pool_select_large_supported(const Geometry &g);
+cudaError_t launch_pool_select_large(const Geometry &g, const LayerTable &layers, const float *raw,
+                                     float *pooled, int32_t *idx, cudaStream_t stream);
 // Block-granular selection (g.select_block >= 2) from final scores [U][P].
 cudaError_t launch_block_select(const Geometry &g, const LayerTable &layers, const float *scores,
                                 int32_t *idx, cudaStream_t stream);

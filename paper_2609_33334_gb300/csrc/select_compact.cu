@@ -119,19 +119,30 @@ struct SelScratch {
 // serialise.  The passes stop early when every key of the selected bin is kept (its count is
 // the rank still wanted): T is then the bin's lowest possible key (the prefix, lower bits
 // zero) and need_eq = C, which keeps exactly the keys >= T.  After two 11-bit passes the bin
-// nearly always holds one key, so the third pass is skipped.  Called by every thread of a
-// block of kSelThreads.
-template <typename KeyAt>
+// nearly always holds one key, so the third pass is skipped.  kBatch > 1 (keys in global
+// memory): each thread loads kBatch keys before it uses any, so their latencies overlap
+// instead of adding up between the shared-memory atomics.  Called by every thread of a block
+// of kSelThreads.
+template <int kBatch = 1, typename KeyAt>
 __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, uint32_t &T,
                                 int &need_eq, uint32_t kmin = 0xffffffffu, uint32_t kmax = 0u,
                                 bool have_range = false)
 {
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (!have_range)
-        for (int j = tid; j < C; j += kSelThreads) {
-            const uint32_t k = key_at(j);
-            kmin = min(kmin, k);
-            kmax = max(kmax, k);
+        for (int j0 = tid; j0 < C; j0 += kBatch * kSelThreads) {
+            uint32_t kb[kBatch];
+#pragma unroll
+            for (int q = 0; q < kBatch; ++q) {
+                const int j = j0 + q * kSelThreads;
+                kb[q] = j < C ? key_at(j) : 0u;
+            }
+#pragma unroll
+            for (int q = 0; q < kBatch; ++q)
+                if (j0 + q * kSelThreads < C) {
+                    kmin = min(kmin, kb[q]);
+                    kmax = max(kmax, kb[q]);
+                }
         }
     kmin = __reduce_min_sync(0xffffffffu, kmin);
     kmax = __reduce_max_sync(0xffffffffu, kmax);
@@ -166,10 +177,17 @@ __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, u
         for (int i = tid; i < kRadixBins; i += kSelThreads)
             sc.hist[i] = 0;
         __syncthreads();
-        for (int j = tid; j < C; j += kSelThreads) {
-            const uint32_t k = key_at(j);
-            if ((k & mask) == prefix)
-                atomicAdd(&sc.hist[(k >> shift) & bmask], 1u);
+        for (int j0 = tid; j0 < C; j0 += kBatch * kSelThreads) {
+            uint32_t kb[kBatch];
+#pragma unroll
+            for (int q = 0; q < kBatch; ++q) {
+                const int j = j0 + q * kSelThreads;
+                kb[q] = j < C ? key_at(j) : 0u;
+            }
+#pragma unroll
+            for (int q = 0; q < kBatch; ++q)
+                if (j0 + q * kSelThreads < C && (kb[q] & mask) == prefix)
+                    atomicAdd(&sc.hist[(kb[q] >> shift) & bmask], 1u);
         }
         __syncthreads();
         {
@@ -225,8 +243,9 @@ __device__ void radix_threshold(KeyAt key_at, int C, int keep, SelScratch &sc, u
 // equal to T -- in ascending order to out[0 .. keep).  Warp w walks a contiguous range of the
 // candidates twice: it counts its keys above and equal to T, then (after two scans over the
 // warps) writes its kept positions; the equal keys a warp keeps follow from the equal keys
-// before its range.  Called by every thread of a block of kSelThreads.
-template <typename KeyAt>
+// before its range.  kBatch as for radix_threshold (a warp loads kBatch rows of 32 keys, then
+// uses them in order).  Called by every thread of a block of kSelThreads.
+template <int kBatch = 1, typename KeyAt>
 __device__ void ordered_compaction(KeyAt key_at, int C, uint32_t T, int need_eq, int keep, int s0,
                                    int32_t *out, SelScratch &sc)
 {
@@ -235,11 +254,19 @@ __device__ void ordered_compaction(KeyAt key_at, int C, uint32_t T, int need_eq,
     const int per_w = ((C + kSelWarps - 1) / kSelWarps + 31) & ~31;
     const int w_lo = min(C, warp * per_w), w_hi = min(C, w_lo + per_w);
     int eq_cnt = 0, gt_cnt = 0;
-    for (int c = w_lo; c < w_hi; c += 32) {
-        const int j = c + lane;
-        const uint32_t k = j < w_hi ? key_at(j) : 0u;
-        eq_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k == T));
-        gt_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && k > T));
+    for (int c0 = w_lo; c0 < w_hi; c0 += 32 * kBatch) {
+        uint32_t kb[kBatch];
+#pragma unroll
+        for (int q = 0; q < kBatch; ++q) {
+            const int j = c0 + 32 * q + lane;
+            kb[q] = j < w_hi ? key_at(j) : 0u;
+        }
+#pragma unroll
+        for (int q = 0; q < kBatch; ++q) {
+            const int j = c0 + 32 * q + lane;
+            eq_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && kb[q] == T));
+            gt_cnt += __popc(__ballot_sync(0xffffffffu, j < w_hi && kb[q] > T));
+        }
     }
     if (lane == 0) {
         sc.warp_a[warp] = eq_cnt;
@@ -257,18 +284,28 @@ __device__ void ordered_compaction(KeyAt key_at, int C, uint32_t T, int need_eq,
     scan_warp_counts(sc.warp_a, sc.warp_c);
     __syncthreads();
     int sel_run = sc.warp_c[warp], eq_run = eq_base;
-    for (int c = w_lo; c < w_hi; c += 32) {
-        const int j = c + lane;
-        const uint32_t k = j < w_hi ? key_at(j) : 0u;
-        const bool eq = j < w_hi && k == T;
-        const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
-        const bool sel = j < w_hi && (k > T || (eq && eq_run + __popc(eqb & lt_mask) < need_eq));
-        const uint32_t selb = __ballot_sync(0xffffffffu, sel);
-        const int pos = sel_run + __popc(selb & lt_mask);
-        if (sel && pos < keep)
-            out[pos] = s0 + j;
-        sel_run += __popc(selb);
-        eq_run += __popc(eqb);
+    for (int c0 = w_lo; c0 < w_hi; c0 += 32 * kBatch) {
+        uint32_t kb[kBatch];
+#pragma unroll
+        for (int q = 0; q < kBatch; ++q) {
+            const int j = c0 + 32 * q + lane;
+            kb[q] = j < w_hi ? key_at(j) : 0u;
+        }
+#pragma unroll
+        for (int q = 0; q < kBatch; ++q) {
+            const int j = c0 + 32 * q + lane;
+            const uint32_t k = kb[q];
+            const bool eq = j < w_hi && k == T;
+            const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+            const bool sel =
+                j < w_hi && (k > T || (eq && eq_run + __popc(eqb & lt_mask) < need_eq));
+            const uint32_t selb = __ballot_sync(0xffffffffu, sel);
+            const int pos = sel_run + __popc(selb & lt_mask);
+            if (sel && pos < keep)
+                out[pos] = s0 + j;
+            sel_run += __popc(selb);
+            eq_run += __popc(eqb);
+        }
     }
 }
 
@@ -381,11 +418,12 @@ select_kernel(const float *__restrict__ scores, int32_t *__restrict__ idx, Selec
 
     uint32_t T;
     int need_eq;
-    radix_threshold(key_at, C, keep, scr, T, need_eq);
+    constexpr int kBatch = SMEM ? 1 : 8;   // keys in global memory: batched loads
+    radix_threshold<kBatch>(key_at, C, keep, scr, T, need_eq);
     if (C <= 32 * kSelThreads)
         ordered_compaction_masks(key_at, C, T, need_eq, keep, s0, out + s0, scr);
     else
-        ordered_compaction(key_at, C, T, need_eq, keep, s0, out + s0, scr);
+        ordered_compaction<kBatch>(key_at, C, T, need_eq, keep, s0, out + s0, scr);
 }
 
 cudaError_t launch_select(const Geometry &g, const LayerTable &layers, const float *scores,
@@ -628,6 +666,125 @@ cudaError_t launch_pool_select(const Geometry &g, const LayerTable &layers, cons
     if (err != cudaSuccess)
         return err;
     kern<<<(unsigned)g.U, kPsThreads, smem, stream>>>(raw, pooled_out, idx, p, g.pool_kernel);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Pooling and selection fused for rows longer than kPsMaxP (the 128K-key caches), where the
+// keys do not fit in shared memory: one CTA per unit pools its row tile by tile through
+// shared memory (kPlTile positions and kPsGuard guard cells of the pool's neutral value on
+// each side, the same arithmetic and order as pool_kernel, so the pooled values are
+// bit-identical), writes the pooled row out and tracks the candidates' key range on the way,
+// then runs the radix select and the ordered compaction on keys read back from global memory
+// (L2: the CTA has just written them), kBatch at a time.  This replaces pool_kernel plus
+// select_kernel, whose selection read each key with its own memory latency.
+
+constexpr int kPlTile = 32768;   // positions pooled per shared-memory tile (128 KB)
+
+template <int POOL, int R>
+__global__ void __launch_bounds__(kSelThreads, 1)
+pool_select_large_kernel(const float *__restrict__ raw, float *pooled, int32_t *__restrict__ idx,
+                         SelectParams p, int kernel)
+{
+    extern __shared__ __align__(16) float stile[];   // [kPsGuard][kPlTile][kPsGuard]
+    __shared__ SelScratch sc;
+
+    const int tid = threadIdx.x;
+    const int64_t u = blockIdx.x;
+    const Geometry &g = p.g;
+    int budget;
+    int32_t *out = idx + unit_row_base(p, u, budget);
+    const int P = g.P, s0 = g.sinks, tail = g.n - g.P;
+    const int C = P - s0;                    // candidates [s0, P)
+    const int keep = budget - s0 - tail;     // candidates to keep
+    const float *row = raw + u * (int64_t)P;
+    float *prow = pooled + u * (int64_t)P;
+    const int r = R >= 0 ? R : kernel / 2;   // <= kPsGuard (the launcher checks)
+    const float neutral = POOL == DGE_POOL_MAX ? -INFINITY : 0.f;
+    const float inv_kernel = 1.0f / (float)kernel;
+
+    uint32_t kmin = 0xffffffffu, kmax = 0u;   // range of the candidate keys [s0, P)
+    for (int t0 = 0; t0 < P; t0 += kPlTile) {
+        const int len = min(kPlTile, P - t0);
+        for (int i = tid; i < len + 2 * kPsGuard; i += kSelThreads) {
+            const int j = t0 - kPsGuard + i;
+            stile[i] = j >= 0 && j < P ? row[j] : neutral;
+        }
+        __syncthreads();
+        for (int i = tid; i < len; i += kSelThreads) {
+            const float *w = stile + kPsGuard + i;
+            float x = neutral;
+            if (R > 0) {
+#pragma unroll
+                for (int q = -(R > 0 ? R : 0); q <= (R > 0 ? R : 0); ++q)
+                    x = POOL == DGE_POOL_MAX ? fmaxf(x, w[q]) : x + w[q];
+            } else {
+                for (int q = -r; q <= r; ++q)
+                    x = POOL == DGE_POOL_MAX ? fmaxf(x, w[q]) : x + w[q];
+            }
+            if (POOL == DGE_POOL_AVG)
+                x *= inv_kernel;
+            const int j = t0 + i;
+            prow[j] = x;
+            if (j >= s0) {
+                const uint32_t k = float_key(x);
+                kmin = min(kmin, k);
+                kmax = max(kmax, k);
+            }
+        }
+        __syncthreads();   // the tile is read before the next one overwrites it
+    }
+
+    for (int j = tid; j < s0; j += kSelThreads)
+        out[j] = j;
+    for (int j = tid; j < tail; j += kSelThreads)
+        out[s0 + keep + j] = P + j;
+    if (keep <= 0)
+        return;
+    if (keep >= C) {
+        for (int j = tid; j < C; j += kSelThreads)
+            out[s0 + j] = s0 + j;
+        return;
+    }
+    // Keys from the pooled row this CTA has just written: loads through L2 (ld.global.cg),
+    // never the read-only path, which need not see this kernel's own stores.
+    const float *keys = prow + s0;
+    auto key_at = [&](int j) -> uint32_t { return float_key(__ldcg(keys + j)); };
+    uint32_t T;
+    int need_eq;
+    radix_threshold<8>(key_at, C, keep, sc, T, need_eq, kmin, kmax, true);
+    if (C <= 32 * kSelThreads)
+        ordered_compaction_masks(key_at, C, T, need_eq, keep, s0, out + s0, sc);
+    else
+        ordered_compaction<8>(key_at, C, T, need_eq, keep, s0, out + s0, sc);
+}
+
+bool pool_select_large_supported(const Geometry &g)
+{
+    return g.P > kPsMaxP && (g.pool == DGE_POOL_AVG || g.pool == DGE_POOL_MAX) &&
+           g.pool_kernel >= 1 && g.pool_kernel / 2 <= kPsGuard;
+}
+
+cudaError_t launch_pool_select_large(const Geometry &g, const LayerTable &layers, const float *raw,
+                                     float *pooled, int32_t *idx, cudaStream_t stream)
+{
+    SelectParams p;
+    p.g = g;
+    p.layers = layers;
+    const size_t smem = (size_t)(kPlTile + 2 * kPsGuard) * sizeof(float);
+    using KernT = void (*)(const float *, float *, int32_t *, SelectParams, int);
+    KernT kern;
+    if (g.pool == DGE_POOL_MAX)
+        kern = g.pool_kernel == 7 ? pool_select_large_kernel<DGE_POOL_MAX, 3>
+                                  : pool_select_large_kernel<DGE_POOL_MAX, -1>;
+    else
+        kern = g.pool_kernel == 7 ? pool_select_large_kernel<DGE_POOL_AVG, 3>
+                                  : pool_select_large_kernel<DGE_POOL_AVG, -1>;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem);
+    if (err != cudaSuccess)
+        return err;
+    kern<<<(unsigned)g.U, kSelThreads, smem, stream>>>(raw, pooled, idx, p, g.pool_kernel);
     return cudaGetLastError();
 }
 

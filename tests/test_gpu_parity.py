@@ -68,6 +68,10 @@ SMALL = {
     "sinks_scored": WL["c1_tiny"].with_(sinks=4, budgets=(100,)),
     "no_pool": WL["c1_tiny"].with_(pool=inputs.POOL_NONE, pool_kernel=1),
     "long_p": WL["c1_tiny"].with_(n=33500, budgets=(600,), n_spans=0),  # P > 32768
+    # longer rows pool tile by tile (32768 positions a tile): avg-7 over two tiles, and max-5
+    # (radius known only at run time) over three
+    "long_p_avg": WL["c1_tiny"].with_(n=33500, budgets=(600,), n_spans=0, pool=inputs.POOL_AVG),
+    "long_p_max5": WL["c1_tiny"].with_(n=70000, budgets=(2000,), n_spans=0, pool_kernel=5),
     # the fused pooling reads whole 128-position chunks: P = 32768 exactly (the largest fused
     # row, no partial chunk) and P = 129 (one chunk and one position)
     "p_32768": WL["c1_tiny"].with_(n=32778, budgets=(700,), n_spans=0),
@@ -127,13 +131,14 @@ def test_runs_are_bit_identical():
 
 
 @pytest.mark.parametrize("name", ["c2_small", "c3_small", "no_pool", "keep_none", "keep_all",
-                                  "long_p", "p_32768", "p_32768_avg", "p_129"])
+                                  "long_p", "long_p_avg", "long_p_max5", "p_32768",
+                                  "p_32768_avg", "p_129"])
 def test_separate_calls_match_fused(name):
     """dge_score -> dge_select -> dge_compact equals dge_evict, bit for bit.
 
-    dge_evict pools and selects in one kernel (P <= 32768) while the separate calls run the
-    pooling and selection kernels; max-, avg- and no pooling, the degenerate budgets, and a
-    case through the larger-P path."""
+    dge_evict pools and selects in one kernel (one for P <= 32768, one for longer rows) while
+    the separate calls run the pooling and selection kernels; max-, avg- and no pooling, the
+    degenerate budgets, and rows longer than 32768 positions."""
     wl = SMALL[name]
     tens, fused = run(wl)
     p = api.problem_from_workload(wl)
