@@ -84,6 +84,7 @@ constexpr int kLagGridX10 = DGE_TC_LAG_GRID_X10;
 #endif
 constexpr int kClaimAhead = DGE_TC_CLAIM_AHEAD;
 constexpr int kChunkTiles = DGE_TC_CHUNK_TILES;
+constexpr int kPageBuf = tc::kPageWindow + 4;   // ints of one page-id window buffer
 // Fewest items (unit, chunk) of a launch of whole units: about three per SM of a 152-SM GB300.
 constexpr int kMinItems = 456;
 // Arrivals that free a ring slot: the MMA warp, the two coordinator warps, the epilogue warps.
@@ -221,7 +222,7 @@ struct Smem {
     float *red;          // [2][kEpiWG][4][kMaxGroups * 16] per-warp phase-1 row sums
     int *sLbad;          // [2] that task's unit is recomputed elsewhere
     float *xch;          // [kAccBufs][kEpiWG][128] phase-2 partial column sums
-    int *pages;          // [tc::kPageWindow + 4] page ids of the producer's window (paged caches)
+    int *pages;          // [2][kPageBuf] page ids of the producer's current and next window (paged caches)
 };
 
 __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
@@ -232,7 +233,7 @@ __host__ __device__ inline size_t smem_bytes(int r_pad, int nslab, int kstages)
            + kStageBytes                          // lse merge staging
            + kCtrlBytes                           // barriers, tmem holder, flags
            + (2 * 256 + 2 * kEpiWG * 4 * kMaxGroups * 16) * 4 + 16
-           + kAccBufs * kEpiWG * kTile * 4 + (tc::kPageWindow + 4) * 4;
+           + kAccBufs * kEpiWG * kTile * 4 + 2 * kPageBuf * 4;
 }
 
 __device__ __forceinline__ Smem carve(uint8_t *raw, int r_pad, int nslab, int kstages)
@@ -517,13 +518,32 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                     nq = true;
                 }
                 if constexpr (kPaged) {
-                    if (tile % tc::kPageWindowTiles == 0) {
-                        w0 = T.k_lo + tile * kTile;
-                        if (lane == 0)
-                            tc::fetch_pages(sm.pages, a.kp, bb, w0,
-                                            min(T.ntiles - tile, tc::kPageWindowTiles));
+                    // Page ids a window of kPageWindowTiles tiles at a time, double buffered:
+                    // at a window's first tile the next window's ids are requested into the
+                    // other buffer (whose window is done), and only this window's are waited
+                    // for -- in flight since the previous window began, except for a task's
+                    // first window.
+                    constexpr int W = tc::kPageWindowTiles;
+                    if (tile % W == 0) {
+                        const int wi = tile / W;
+                        int *buf = sm.pages + (wi & 1) * kPageBuf;
+                        if (wi == 0) {
+                            tc::fetch_pages_issue_warp(buf, a.kp, bb, T.k_lo, min(T.ntiles, W),
+                                                       lane);
+                            tc::fetch_pages_commit();
+                        }
+                        if (tile + W < T.ntiles) {
+                            tc::fetch_pages_issue_warp(sm.pages + ((wi + 1) & 1) * kPageBuf,
+                                                       a.kp, bb, T.k_lo + (tile + W) * kTile,
+                                                       min(T.ntiles - tile - W, W), lane);
+                            tc::fetch_pages_commit();
+                            tc::fetch_pages_wait_group<1>();
+                        } else {
+                            tc::fetch_pages_wait_group<0>();
+                        }
                         __syncwarp();
-                        ids = tc::page_ids_at(sm.pages, a.kp, bb, w0);
+                        w0 = T.k_lo + tile * kTile;
+                        ids = tc::page_ids_at(buf, a.kp, bb, w0);
                     }
                 }
                 long long c0 = tclock<kTr>();
@@ -564,6 +584,8 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             p = np;
             q_ready = nq;
         }
+        if constexpr (kPaged)
+            tc::fetch_pages_wait_group<0>();   // no page-id copy outlives the loop (aborts)
         if (lane == 0) {
             trace_put<kTr>(a, kTrProdWaitQ, cy_wq);
             trace_put<kTr>(a, kTrProdWaitK, cy_wk);
