@@ -496,6 +496,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
             const uint64_t pol = T.phase == 2 ? drop : keep;
             int w0 = 0;               // first key of the page-id window (paged caches)
             const int *ids = sm.pages;
+            int wrun = -1;            // lane t: tile t of the window as one run of pages, or -1
             for (int tile = 0; tile < T.ntiles; ++tile) {
                 if (tile == claim_at) {
                     if (lane == 0)
@@ -544,6 +545,7 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                         __syncwarp();
                         w0 = T.k_lo + tile * kTile;
                         ids = tc::page_ids_at(buf, a.kp, bb, w0);
+                        wrun = tc::tile_runs(a.kp, ids, w0, min(T.ntiles - tile, W), lane);
                     }
                 }
                 long long c0 = tclock<kTr>();
@@ -563,7 +565,10 @@ score_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__
                 tc::load_k_tile_warp<kPaged>(sm.k + (size_t)ks * a.nslab * kSlabBytes,
                                              kSlabBytes, a.nslab, &tmK, &tmKm,
                                              &sm.bar[kBarKFull + ks], T.k_lo + tile * kTile, l,
-                                             bb, h, a.kp, ids, w0, pol, lane);
+                                             bb, h, a.kp, ids, w0, pol, lane,
+                                             kPaged ? __shfl_sync(0xffffffffu, wrun,
+                                                                  tile % tc::kPageWindowTiles)
+                                                    : -1);
                 if (++ks == a.kstages) {
                     ks = 0;
                     kph ^= 1;

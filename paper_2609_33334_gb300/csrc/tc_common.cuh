@@ -181,6 +181,28 @@ __device__ __forceinline__ void fetch_pages_wait_group()
     asm volatile("cp.async.wait_group %0;" ::"n"(pending) : "memory");
 }
 
+// For the window of kPageWindowTiles (= 32) tiles from key w0 (ids from fetch_pages): lane t
+// returns the first page of tile t when that tile's pages are consecutive and the merged map
+// can load it as one box a slab, else -1.  Every lane of the warp calls it once a window, so
+// the per-tile path reads one register (a shuffle) instead of the tile's page ids.
+__device__ __forceinline__ int tile_runs(const KPaging &pg, const int *ids, int w0, int tiles,
+                                         int lane)
+{
+    static_assert(kPageWindowTiles == 32, "one lane per tile of the window");
+    if (!pg.merged || pg.page_size >= 128 || lane >= tiles)
+        return -1;
+    const int npg = 128 >> pg.ps_shift;
+    const int k0 = w0 + lane * 128;
+    const int valid = (pg.n - k0 + pg.page_size - 1) >> pg.ps_shift;
+    if (valid < npg)
+        return -1;
+    const int first = ids[lane * npg];
+    bool run = (unsigned)first <= (unsigned)(pg.num_pages - npg);
+    for (int j = 1; j < npg; ++j)
+        run = run && ids[lane * npg + j] == first + j;
+    return run ? first : -1;
+}
+
 // Where fetch_pages(buf, pg, bb, k0, ...) puts the page ids (any thread can compute it).
 __device__ __forceinline__ const int *page_ids_at(int *buf, const KPaging &pg, int bb, int k0)
 {
@@ -263,13 +285,16 @@ __device__ __forceinline__ void load_k_tile(uint8_t *dst, uint32_t slab_bytes, i
 // load_k_tile issued by a whole warp, one box per lane: box i of a tile is slab i % nslab of
 // page i / nslab (nslab boxes for a contiguous cache, a page of 128 slots or more, or a run
 // of consecutive pages).  The caller arms `bar` for the whole tile before any lane issues.
+// Pages below 128 slots: run_first >= 0 says the tile's pages are consecutive from page
+// run_first (the merged map applies; the caller decides, see tile_runs), else one box per
+// page and slab.
 template <bool kPaged>
 __device__ __forceinline__ void load_k_tile_warp(uint8_t *dst, uint32_t slab_bytes, int nslab,
                                                  const CUtensorMap *map,
                                                  const CUtensorMap *merged, uint64_t *bar,
                                                  int k0, int l, int bb, int h, const KPaging &pg,
                                                  const int *ids, int w0, uint64_t policy,
-                                                 int lane)
+                                                 int lane, int run_first = -1)
 {
     if constexpr (!kPaged) {
         if (lane < nslab)
@@ -290,17 +315,11 @@ __device__ __forceinline__ void load_k_tile_warp(uint8_t *dst, uint32_t slab_byt
         const int npg = 128 >> pg.ps_shift;
         const int i0 = (k0 - w0) >> pg.ps_shift;
         const int valid = (pg.n - k0 + pg.page_size - 1) >> pg.ps_shift;
-        if (pg.merged && valid >= npg) {
-            const int first = ids[i0];
-            bool run = (unsigned)first <= (unsigned)(pg.num_pages - npg);
-            for (int j = 1; j < npg; ++j)
-                run = run && ids[i0 + j] == first + j;
-            if (run) {
-                if (lane < nslab)
-                    ptx::tma_load_5d_hint(dst + lane * slab_bytes, merged, bar, lane * 64, h,
-                                          first << pg.ps_shift, l, 0, policy);
-                return;
-            }
+        if (run_first >= 0) {   // the tile's pages are consecutive: one box a slab
+            if (lane < nslab)
+                ptx::tma_load_5d_hint(dst + lane * slab_bytes, merged, bar, lane * 64, h,
+                                      run_first << pg.ps_shift, l, 0, policy);
+            return;
         }
         const int j = lane / nslab, s = lane - j * nslab;
         if (j < npg) {
