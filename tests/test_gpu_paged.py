@@ -228,3 +228,21 @@ def test_paged_evict_matches_oracle(name, page_size):
     refs = oracle_units(wl, tens, units)
     for (l, b, h) in units:
         compare_unit(wl, got, tens, l, b, h, ref=refs[(l, b, h)])
+
+
+@pytest.mark.parametrize("page_size,order", [(16, "sequential"), (16, "runs"), (16, "random"),
+                                             (32, "sequential"), (128, "random")])
+def test_paged_tasks_span_page_windows(page_size, order):
+    """Key chunks longer than the producer's page-id window (32 tiles): 128 units of 32768
+    positions take chunks of 64 tiles, so each task reads two windows, the second one's ids
+    fetched while the first is in use, and the consecutive-pages check runs per window.  The
+    outputs equal the contiguous run's."""
+    wl = WL["c3_8b_32k_pyramid"].with_(L=4, b=4, budgets=(2048, 1024, 512, 256), n_spans=16)
+    tens = inputs.make_inputs(wl, device="cuda")
+    p = api.problem_from_workload(wl)
+    ref = api.evict(p, tens["K"], tens["V"], tens["Q"], want_scores=True)
+    K, V, pg = _paged(tens, page_size, seed=5, order=order)
+    got = api.evict(p, K, V, tens["Q"], want_scores=True, paging=pg)
+    torch.cuda.synchronize()
+    for k in ("idx", "Kc", "Vc", "scores"):
+        assert torch.equal(got[k], ref[k]), k
