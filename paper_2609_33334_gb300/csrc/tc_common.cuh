@@ -303,8 +303,11 @@ __device__ __forceinline__ void load_k_tile_warp(uint8_t *dst, uint32_t slab_byt
     } else if (pg.page_size >= 128) {
         int page = 0, slot = 0;
         if (k0 < pg.n) {
-            const int pi = k0 / pg.page_size;
-            const int pid = ids[pi - w0 / pg.page_size];
+            // Power-of-two page sizes by shifts (off the producer's path), others by division.
+            const bool pow2 = (1 << pg.ps_shift) == pg.page_size;
+            const int pi = pow2 ? k0 >> pg.ps_shift : k0 / pg.page_size;
+            const int pw = pow2 ? w0 >> pg.ps_shift : w0 / pg.page_size;
+            const int pid = ids[pi - pw];
             page = (unsigned)pid < (unsigned)pg.num_pages ? pid : 0;
             slot = k0 - pi * pg.page_size;
         }
@@ -321,7 +324,8 @@ __device__ __forceinline__ void load_k_tile_warp(uint8_t *dst, uint32_t slab_byt
                                       run_first << pg.ps_shift, l, 0, policy);
             return;
         }
-        const int j = lane / nslab, s = lane - j * nslab;
+        // nslab is 1 or 2 (d = 64 or 128): a shift, not a division, on the producer's path.
+        const int j = lane >> (nslab - 1), s = lane & (nslab - 1);
         if (j < npg) {
             int page = 0;
             if (j < valid) {
