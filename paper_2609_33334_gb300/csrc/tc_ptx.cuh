@@ -73,15 +73,19 @@ __device__ __forceinline__ bool mbar_test_token(uint64_t *bar, uint64_t state)
 // Test for completion of the phase with parity `parity`; the thread may be suspended in
 // hardware (up to a time hint of about a millisecond) until the phase completes, so waiting
 // warps do not spin on the issue slots.
+// One bounded-time probe of an mbarrier phase (the thread may be suspended for a
+// system-defined interval while the phase is incomplete).  No suspend-time hint: with a 1 ms
+// hint the waiting warps resumed later after the phase completed, measured 2-3 % slower in
+// the scoring kernel (c3 2.476 -> 2.426 ms, c5 16 layers 4.751 -> 4.603 ms without it).
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
 {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
         "selp.b32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(smem_addr(bar)), "r"(parity), "r"(1000000u)
+        : "r"(smem_addr(bar)), "r"(parity)
         : "memory");
     return ok != 0;
 }
