@@ -53,3 +53,33 @@ def test_c5_flops_and_slm_floor():
     slm = WL["c5_slm"]
     assert bench.step_bytes(slm) == pytest.approx(2.68e9, rel=2e-3)
     assert bench.tokens_per_step(slm) == 10_485_760
+
+
+def test_traffic_digest_follows_the_kernels_own_source(tmp_path, monkeypatch):
+    """An ncu traffic figure stays valid while its kernel's own source and the shared headers
+    are unchanged, whatever happens to another kernel's file, and is voided by either."""
+    csrc = tmp_path / "paper_2609_33334_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (tmp_path / "include").mkdir()
+    (tmp_path / "include" / "dge.h").write_text("// api\n")
+    (tmp_path / "profiles").mkdir()
+    for name, text in (("score_tc.cu", "a"), ("select_compact.cu", "b"), ("h2o_tc.cu", "c"),
+                       ("common.cuh", "h")):
+        (csrc / name).write_text(text)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    d_tc = bench.source_digest("score_tc")
+    (tmp_path / "profiles" / "dram_traffic.txt").write_text(
+        f"# header\nscore_tc c3_8b_32k_pyramid 123 {d_tc}\n")
+    assert bench.ncu_traffic("score_tc", "c3_8b_32k_pyramid") == 123.0
+    assert bench.ncu_traffic("score_tc", "c2_8b_8k") is None           # another workload
+    (csrc / "select_compact.cu").write_text("b2")                        # another kernel's file
+    assert bench.source_digest("score_tc") == d_tc
+    assert bench.ncu_traffic("score_tc", "c3_8b_32k_pyramid") == 123.0
+    (csrc / "score_tc.cu").write_text("a2")                              # its own file
+    assert bench.ncu_traffic("score_tc", "c3_8b_32k_pyramid") is None
+    (csrc / "score_tc.cu").write_text("a")
+    assert bench.ncu_traffic("score_tc", "c3_8b_32k_pyramid") == 123.0
+    (csrc / "common.cuh").write_text("h2")                               # a shared header
+    assert bench.ncu_traffic("score_tc", "c3_8b_32k_pyramid") is None
+    # the two H2O launches are one source file: one digest
+    assert bench.source_digest("h2o_tc_lse") == bench.source_digest("h2o_tc_colsum")
